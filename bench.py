@@ -1,0 +1,644 @@
+#!/usr/bin/env python
+"""Benchmark of the GB300 ReSA decode-attention path (one JSON line).
+
+Workload (default ``qwen7b_b8_ctx32k_f32``): one attention layer of
+Qwen2.5-7B geometry (28 query / 4 KV heads, head dim 128, bf16), batch 8,
+32K-token context, block size 16, 10% of blocks kept (min 128 blocks, 1
+forced local block), rectification every f = 32 steps, K with log-normal
+per-channel outlier scales. Synthetic seeded data; no weights.
+
+One benchmark STEP is one rectification period of the path (Algorithm 1):
+f decode steps, each = commit the new token's K/V (+ summary update) ->
+select blocks (Eq. 4/5) -> split-K sparse decode + combine (Algorithm 2),
+then the dense rectification of those f tokens + overwrite commit. To keep
+the HBM numbers honest the step runs over R independent layer caches in
+rotation (the decode steps of one layer are separated by the other layers'
+traffic, as in a model's layer loop); ``value`` is layer-tokens per second
+(tokens pushed through one attention layer of the workload per second).
+
+Timing: W warm-up steps, then K steps replayed from one CUDA graph per step,
+timed with CUDA events on the replay stream between a barrier +
+synchronize on both sides; max over ranks. Per-call durations for the
+roofline come from one CUDA graph per call type holding the step's calls of
+that type in step order, timed with CUDA events (total / calls).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2506_04108_gb300 import synth  # noqa: E402
+
+METRIC = "decode attention tokens/s"
+UNIT = "tokens/s"
+DEFAULT_WORKLOAD = "qwen7b_b8_ctx32k_f32"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+HEAD_DIM = 128
+BLOCK = 16
+
+
+# ------------------------------------------------------------ algorithmic work
+def budget(M: int, keep: float, n_min: int, n_local: int) -> int:
+    return min(M, max(n_min, math.ceil(M * keep), n_local))
+
+
+def decode_bytes(B, Hq, Hkv, T, keep, n_min, n_local) -> int:
+    """Bytes one sparse-decode call must move: K+V of the attended tokens
+    (selected blocks, the partial last block counted by its valid tokens),
+    the queries in and the outputs out."""
+    M = (T + BLOCK - 1) // BLOCK
+    n = budget(M, keep, n_min, n_local)
+    tokens = (n - 1) * BLOCK + (T - BLOCK * (M - 1))
+    return B * Hkv * tokens * 2 * HEAD_DIM * 2 + 2 * B * Hq * HEAD_DIM * 2
+
+
+def select_bytes(B, Hq, Hkv, T, keep, n_min, n_local) -> int:
+    """Summaries read (Eq. 4 reads k_min and k_max of every block), fp32 scores
+    written and read back, queries read, indices written."""
+    M = (T + BLOCK - 1) // BLOCK
+    n = budget(M, keep, n_min, n_local)
+    return B * Hkv * M * 2 * HEAD_DIM * 2 + B * Hkv * M * 8 + B * Hq * HEAD_DIM * 2 + B * Hkv * n * 4
+
+
+def commit_bytes(B, Hkv, n_tokens) -> int:
+    """New K/V read and written, plus one summary read+write per touched block."""
+    return B * Hkv * n_tokens * HEAD_DIM * 2 * 2 * 2 + B * Hkv * 2 * (2 * HEAD_DIM * 2)
+
+
+def rectify_bytes(B, Hq, Hkv, T, f) -> int:
+    """K+V of all T positions per (sequence, KV head), queries in, outputs out."""
+    return B * Hkv * T * 2 * HEAD_DIM * 2 + 2 * B * f * Hq * HEAD_DIM * 2
+
+
+def rectify_flops(B, Hq, T, f) -> int:
+    """Useful causal pairs only: 4 * d flops per (query head, visible key)."""
+    return 4 * HEAD_DIM * Hq * B * (f * T - f * (f - 1) // 2)
+
+
+def eq6_ratio(b: int, keep: float, f: int) -> float:
+    """Eq. 6's memory ratio of the step relative to dense decoding."""
+    return 1.0 / b + keep + 1.0 / f
+
+
+# ------------------------------------------------------------------ helpers
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as fh:
+            return json.load(fh), "measured"
+    return FALLBACK_PEAKS, "fallback"
+
+
+def source_hash(*names) -> str:
+    h = hashlib.sha256()
+    for n in names:
+        with open(os.path.join(ROOT, "paper_2506_04108_gb300", "csrc", n), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(kernel: str, workload: str, src_hash: str):
+    """DRAM bytes per launch of `kernel` from a committed ncu summary, if its
+    recorded source hash still matches the kernel source; else None."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as fh:
+        table = json.load(fh)
+    e = table.get(kernel, {}).get(workload)
+    if not e or e.get("source_hash") != src_hash:
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during the timed region."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu_index = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        try:
+            fd, self.path = tempfile.mkstemp(prefix="resa_clocks_", suffix=".csv")
+            os.close(fd)
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu_index), f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.fh, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.fh.close()
+
+    def summary(self):
+        if self.proc is None or self.path is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as fh:
+            for line in fh:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for nm, v in zip(names, parts[5:9]):
+                    if v.lower() == "active":
+                        reasons.add(nm)
+        os.unlink(self.path)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# --------------------------------------------------------------- distributed
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def init_dist(backend: str):
+    import torch.distributed as dist
+    rank, world, _ = dist_env()
+    if world > 1 and not dist.is_initialized():
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group(backend=backend, rank=rank, world_size=world)
+    return rank, world
+
+
+def barrier():
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized():
+        dist.barrier()
+
+
+def max_over_ranks(x: float, device=None) -> float:
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def aggregate(units_per_rank: float, seconds_max: float, world: int) -> float:
+    """Whole-job throughput: units processed by all ranks / the slowest rank's time."""
+    return units_per_rank * world / seconds_max
+
+
+# ---------------------------------------------------------------- GPU side
+class LayerCache:
+    """One layer's paged cache plus the device inputs/outputs of one period."""
+
+    def __init__(self, w: synth.Workload, capacity_tokens: int, seed: int, device):
+        import torch
+        from paper_2506_04108_gb300 import resa
+        self.w, self.resa = w, resa
+        B, Hq, Hkv, f = w.batch, w.num_q_heads, w.num_kv_heads, w.f
+        maxb = capacity_tokens // BLOCK
+        gen = synth.rng(seed)
+        pt = synth.page_table(gen, B, maxb)
+        self.cache = resa.PagedKVCache(B, Hq, Hkv, maxb, pt, device=device, zero_pools=False)
+        tg = torch.Generator(device=device)
+        tg.manual_seed(seed)
+        scale = torch.from_numpy(synth.channel_scale(gen, Hkv, HEAD_DIM, w.k_channel_sigma)).to(device)
+        for pool, sc in ((self.cache.k_pool, scale), (self.cache.v_pool, None)):
+            for i in range(0, pool.shape[0], 4096):            # fill in chunks to bound temporaries
+                x = torch.randn(pool[i:i + 4096].shape, generator=tg, device=device)
+                if sc is not None:
+                    x *= sc[None, :, None, :]
+                pool[i:i + 4096].copy_(x)
+        self.cache.seq_lens.fill_(w.context)
+        resa.resa_update_summaries(self.cache.struct, 0, -1)
+        self.p = resa.params(w.keep, w.n_min_blocks, w.n_local_blocks)
+        self.n_cap = resa.resa_max_selected(self.cache.struct, self.p)
+        self.ws_bytes = resa.resa_workspace_size(self.cache.struct, self.n_cap, 0, f)
+        self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=device)
+        self.idx = torch.empty((B, Hkv, self.n_cap), dtype=torch.int32, device=device)
+        self.cnt = torch.empty((B, Hkv), dtype=torch.int32, device=device)
+
+        def rn(*shape, s=1.0):
+            return (torch.randn(shape, generator=tg, device=device) * s).to(torch.bfloat16)
+        dk = rn(f, B, Hkv, HEAD_DIM) * scale[None, None].to(torch.bfloat16)
+        dv = rn(f, B, Hkv, HEAD_DIM)
+        dq = rn(f, B, Hq, HEAD_DIM)
+        noise = synth.SPARSE_ERA_NOISE
+        # per-step inputs of the sparse decode steps (sparse-era K/V and queries)
+        self.q = (dq.float() + noise * torch.randn(dq.shape, generator=tg, device=device)).to(torch.bfloat16)
+        self.k = (dk.float() + noise * torch.randn(dk.shape, generator=tg, device=device)).to(torch.bfloat16)
+        self.v = (dv.float() + noise * torch.randn(dv.shape, generator=tg, device=device)).to(torch.bfloat16)
+        # dense re-encode of the f tokens, [B, f, H, d]
+        self.rq = dq.transpose(0, 1).contiguous()
+        self.rk = dk.transpose(0, 1).contiguous()
+        self.rv = dv.transpose(0, 1).contiguous()
+        self.out = torch.empty((f, B, Hq, HEAD_DIM), dtype=torch.bfloat16, device=device)
+        self.rout = torch.empty((B, f, Hq, HEAD_DIM), dtype=torch.bfloat16, device=device)
+
+    # each call below launches: commit 1 kernel, select 2, decode 2, rectify 2
+    KERNELS_PER_DECODE_STEP = 5
+    KERNELS_PER_RECTIFY = 3
+
+    def commit(self, t):
+        self.resa.resa_commit_kv(self.cache.struct, self.k[t], self.v[t], 1, False)
+
+    def select(self, t):
+        self.resa.resa_select_blocks(self.cache.struct, self.q[t], self.p, self.idx, self.cnt, self.n_cap, self.ws,
+                                     self.ws_bytes)
+
+    def sparse_decode(self, t):
+        self.resa.resa_sparse_decode(self.cache.struct, self.q[t], self.idx, self.cnt, self.n_cap, self.p,
+                                     self.out[t], None, 0, self.ws, self.ws_bytes)
+
+    def rectify_attention(self):
+        self.resa.resa_rectify_attention(self.cache.struct, self.rq, self.rk, self.rv, self.w.f, self.p,
+                                         self.rout, None, self.ws, self.ws_bytes)
+
+    def overwrite(self):
+        self.resa.resa_commit_kv(self.cache.struct, self.rk, self.rv, self.w.f, True)
+
+    def decode(self, t):
+        """One decode step of Algorithm 1 for this layer (commit, select, decode)."""
+        self.commit(t)
+        self.select(t)
+        self.sparse_decode(t)
+
+    def rectify(self):
+        """Rectification branch of Algorithm 1 for this layer."""
+        self.rectify_attention()
+        self.overwrite()
+
+
+def run_period(layers):
+    f = layers[0].w.f
+    for t in range(f):
+        for L in layers:
+            L.decode(t)
+    for L in layers:
+        L.rectify()
+
+
+def host_logical_kv(cache, b: int, T: int):
+    """K, V bits [Hkv, T, d] of sequence b gathered from the device pool."""
+    import torch
+    pt = cache.page_table[b].cpu().numpy()
+    t = np.arange(T)
+    pages = torch.from_numpy(pt[t // BLOCK]).long().to(cache.k_pool.device)
+    rows = torch.from_numpy(t % BLOCK).long().to(cache.k_pool.device)
+    K = cache.k_pool[pages, :, rows, :].transpose(0, 1).contiguous()
+    V = cache.v_pool[pages, :, rows, :].transpose(0, 1).contiguous()
+    to_bits = lambda x: x.cpu().view(torch.int16).numpy().view(np.uint16)  # noqa: E731
+    return to_bits(K), to_bits(V)
+
+
+def bits(t):
+    import torch
+    return t.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
+
+
+# ------------------------------------------------------------ oracle sample
+def oracle_period(sample: dict) -> float:
+    """One rectification period of the fp64 oracle for one sequence of one
+    layer (f decode steps + rectification); returns the seconds it took.
+    The state's prefill summaries are built before the clock starts."""
+    import oracle as O
+    K, V = O.widen_bf16(sample["K"]), O.widen_bf16(sample["V"])
+    Hkv, T0, d = K.shape
+    f = int(sample["f"])
+    st = O.SequenceState(Hkv, T0 + f + BLOCK, d, BLOCK)
+    st.prefill(K, V)
+    p = O.ResaParams(float(sample["keep"]), int(sample["n_min"]), int(sample["n_local"]))
+    q, k, v = (O.widen_bf16(sample[x]) for x in ("q", "k", "v"))
+    rq, rk, rv = (O.widen_bf16(sample[x]) for x in ("rq", "rk", "rv"))
+    t0 = time.perf_counter()
+    for i in range(f):
+        O.sparse_decode_step(st, q[i], k[i], v[i], p)
+    O.rectify_step(st, rq, rk, rv, p)
+    return time.perf_counter() - t0
+
+
+def run_oracle_subprocess(sample: dict, threads: int = 1, repeats: int = 1):
+    """Time oracle_period `repeats` times in a fresh process whose BLAS/OpenMP
+    pools are pinned to `threads` (so `cores` is what the oracle actually
+    used); returns the list of per-repeat seconds."""
+    with tempfile.TemporaryDirectory() as d:
+        path = os.path.join(d, "sample.npz")
+        np.savez(path, **sample)
+        env = dict(os.environ)
+        for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "BLIS_NUM_THREADS"):
+            env[v] = str(threads)
+        r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-worker", path,
+                            "--repeats", str(repeats)], env=env, capture_output=True, text=True, timeout=3600)
+        if r.returncode != 0:
+            raise RuntimeError(f"oracle worker failed: {r.stderr[-2000:]}")
+        return json.loads(r.stdout.strip().splitlines()[-1])["seconds"]
+
+
+def host_sample(w: synth.Workload, context: int):
+    """The oracle's input sample drawn on the host with the workload's recipe:
+    one sequence of one layer at the workload's context, one period of inputs."""
+    inp = synth.decode_inputs(w, context=context, steps=w.f, batch=1)
+    return {"K": inp.prefill_k[0], "V": inp.prefill_v[0], "q": inp.step_q[:, 0], "k": inp.step_k[:, 0],
+            "v": inp.step_v[:, 0], "rq": inp.dense_q[:, 0], "rk": inp.dense_k[:, 0], "rv": inp.dense_v[:, 0],
+            "f": w.f, "keep": w.keep, "n_min": w.n_min_blocks, "n_local": w.n_local_blocks}
+
+
+# ------------------------------------------------------------------- arms
+def run_reference(args, w: synth.Workload):
+    """The oracle as it stands, timed on the host cores: each step is one
+    period of one sequence of one layer (a bounded sample of the workload)."""
+    rank, world, _ = dist_env()
+    if world > 1 and rank != 0:
+        return
+    sample = host_sample(w, w.context)
+    times = run_oracle_subprocess(sample, threads=1, repeats=args.warmup + args.steps)
+    per_step = times[args.warmup:]
+    tot = sum(per_step)
+    value = args.steps * w.f / tot
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": config_of(w, args),
+            "cpu_baseline": {"kind": "oracle", "value": value, "unit": UNIT, "cores": 1,
+                             "sample": f"per step: 1 of {w.batch} sequences, 1 layer, {w.f} decode steps + "
+                                       f"1 rectification at context {w.context} (fp64 numpy, 1 BLAS thread)"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def config_of(w: synth.Workload, args) -> dict:
+    return {"workload": w.name, "batch": w.batch, "context": w.context, "q_heads": w.num_q_heads,
+            "kv_heads": w.num_kv_heads, "head_dim": HEAD_DIM, "block_size": BLOCK, "keep": w.keep,
+            "n_min_blocks": w.n_min_blocks, "n_local_blocks": w.n_local_blocks, "f": w.f,
+            "layers_rotated": args.layers, "step": f"{w.f} decode steps + 1 rectification per layer",
+            "l2": f"{args.layers} independent layer caches rotated per decode step (other layers' traffic "
+                  f"between reuses exceeds the 129 MB L2)", "parallelism": f"replicas x{args.gpus} (weak)"}
+
+
+def capture(fn, device):
+    """CUDA graph of the C-ABI calls `fn` issues (captured on a side stream)."""
+    import torch
+    stream = torch.cuda.Stream(device=device)
+    stream.wait_stream(torch.cuda.current_stream())
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        fn()
+    torch.cuda.synchronize()
+    return graph
+
+
+def time_graph(graph, reps: int) -> float:
+    """Mean seconds of one replay, CUDA events on the replay stream."""
+    import torch
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(reps):
+        graph.replay()
+    b.record()
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / 1e3 / reps
+
+
+def check_device_errors(layers):
+    from paper_2506_04108_gb300 import resa
+    for Lc in layers:
+        code, detail = resa.resa_read_device_error(Lc.cache.struct)
+        if code:
+            raise RuntimeError(f"device error {resa.DEVICE_ERRORS.get(code)} detail {detail}")
+
+
+def run_ours(args, w: synth.Workload):
+    import torch
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    if world > 1:
+        init_dist("nccl")
+    from paper_2506_04108_gb300 import build as _b
+    from paper_2506_04108_gb300 import resa
+    _b.build()
+    resa.load()
+
+    L, f, B = args.layers, w.f, w.batch
+    # periods that append f tokens: warm-up call, graph warm-up/timed/e2e replays, attribution commits
+    periods_total = 1 + args.warmup + args.steps + args.steps + 1 + 2 * ATTR_REPS
+    capacity = ((w.context + f * periods_total + BLOCK) // BLOCK + 1) * BLOCK
+    layers = [LayerCache(w, capacity, w.seed * 100 + 17 * rank + i, device) for i in range(L)]
+    torch.cuda.synchronize()
+    T = w.context                           # tokens in every sequence of every layer
+
+    # warm-up call outside any graph (sets kernel attributes), then capture one step
+    run_period(layers)
+    T += f
+    graph = capture(lambda: run_period(layers), device)
+    for _ in range(args.warmup):
+        graph.replay()
+        T += f
+    torch.cuda.synchronize()
+    check_device_errors(layers)
+
+    # ---- timed region ----
+    T_timed0 = T
+    with ClockSampler(local) as clocks:
+        barrier()
+        torch.cuda.synchronize()
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record()
+        for _ in range(args.steps):
+            graph.replay()
+        s1.record()
+        torch.cuda.synchronize()
+        barrier()
+    T += f * args.steps
+    secs = s0.elapsed_time(s1) / 1e3
+    secs_max = max_over_ranks(secs, device)
+    tokens_per_rank = B * f * L * args.steps
+    value = aggregate(tokens_per_rank, secs_max, world)
+    clk = clocks.summary()
+
+    # ---- end to end through the public API with host buffers ----
+    e2e = run_e2e(args, layers, graph)
+    T += f * args.steps
+
+    # ---- per-call durations: one graph per call type, the period's calls of that type in order ----
+    T_attr = T
+    kinds = {
+        "select": lambda: [Lc.select(t) for t in range(f) for Lc in layers],
+        "decode": lambda: [Lc.sparse_decode(t) for t in range(f) for Lc in layers],
+        "rectify": lambda: [Lc.rectify_attention() for Lc in layers],
+        "overwrite": lambda: [Lc.overwrite() for Lc in layers],
+        "commit": lambda: [Lc.commit(t) for t in range(f) for Lc in layers],
+    }
+    ncalls = {"select": f * L, "decode": f * L, "rectify": L, "overwrite": L, "commit": f * L}
+    mean_us = {}
+    for kind, fn in kinds.items():
+        gk = capture(fn, device)             # capture does not execute
+        gk.replay()                          # warm
+        if kind == "commit":
+            T += f
+        mean_us[kind] = time_graph(gk, ATTR_REPS) / ncalls[kind] * 1e6
+        if kind == "commit":
+            T += f * ATTR_REPS
+        del gk
+    check_device_errors(layers)
+    Tm = T_attr + f // 2
+    algo = {
+        "commit": commit_bytes(B, w.num_kv_heads, 1),
+        "select": select_bytes(B, w.num_q_heads, w.num_kv_heads, Tm, w.keep, w.n_min_blocks, w.n_local_blocks),
+        "decode": decode_bytes(B, w.num_q_heads, w.num_kv_heads, T_attr, w.keep, w.n_min_blocks,
+                               w.n_local_blocks),
+        "rectify": rectify_bytes(B, w.num_q_heads, w.num_kv_heads, T_attr, f),
+        "overwrite": commit_bytes(B, w.num_kv_heads, f),
+    }
+    peaks, peak_kind = load_peaks()
+    hbm = float(peaks["hbm_gbs"])
+    per_step_us = {k: mean_us[k] * ncalls[k] for k in mean_us}
+    tot = sum(per_step_us.values())
+    calls = {}
+    for k in mean_us:
+        gbs = algo[k] / (mean_us[k] * 1e-6) / 1e9
+        calls[k] = {"us_per_call": round(mean_us[k], 2), "calls_per_step": ncalls[k], "GB/s": round(gbs, 1),
+                    "frac_hbm": round(gbs / hbm, 3), "share_of_step": round(per_step_us[k] / tot, 3),
+                    "algorithmic_bytes": int(algo[k])}
+    rflops = rectify_flops(B, w.num_q_heads, T_attr, f)
+    calls["rectify"]["TFLOP/s"] = round(rflops / (mean_us["rectify"] * 1e-6) / 1e12, 1)
+    calls["rectify"]["frac_bf16_sustained"] = round(rflops / (mean_us["rectify"] * 1e-6) / 1e12 /
+                                                    float(peaks["bf16_tflops_sustained"]), 3)
+    dominant = max(per_step_us, key=per_step_us.get)
+    kernel, src = {"decode": ("sparse_decode_kernel", "sparse_decode.cu"), "select": ("topn_kernel", "select.cu"),
+                   "rectify": ("rectify_kernel", "rectify.cu"), "commit": ("commit_append_kernel", "kv_commit.cu"),
+                   "overwrite": ("commit_overwrite_kernel", "kv_commit.cu")}[dominant]
+    achieved = algo[dominant] / (mean_us[dominant] * 1e-6) / 1e9
+    roofline = {"bound": "hbm", "call": dominant, "kernel": kernel, "achieved": round(achieved, 1), "peak": hbm,
+                "unit": "GB/s", "frac": round(achieved / hbm, 3), "peak_kind": peak_kind,
+                "traffic": profiled_traffic(kernel, w.name, source_hash(src)),
+                "algorithmic_bytes_per_launch": int(algo[dominant]),
+                "timing": "CUDA events around a graph of the step's calls of this kind; per call = total / calls"}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        Kb, Vb = host_logical_kv(layers[0].cache, 0, w.context)
+        sample = {"K": Kb, "V": Vb, "q": bits(layers[0].q[:, 0]), "k": bits(layers[0].k[:, 0]),
+                  "v": bits(layers[0].v[:, 0]), "rq": bits(layers[0].rq[0]), "rk": bits(layers[0].rk[0]),
+                  "rv": bits(layers[0].rv[0]), "f": f, "keep": w.keep, "n_min": w.n_min_blocks,
+                  "n_local": w.n_local_blocks}
+        secs_cpu = run_oracle_subprocess(sample, threads=1)[0]
+        cpu = {"value": round(f / secs_cpu, 2), "unit": UNIT, "cores": 1, "kind": "oracle",
+               "sample": f"1 of {B} sequences x 1 of {L} layers: {f} decode steps + 1 rectification at context "
+                         f"{w.context} (fp64 numpy, 1 BLAS thread)", "seconds": round(secs_cpu, 3)}
+
+    launches = args.steps * L * (f * LayerCache.KERNELS_PER_DECODE_STEP + LayerCache.KERNELS_PER_RECTIFY)
+    line = {"metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(secs_max * 1e3 / args.steps, 4), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": config_of(w, args), "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": launches, "clocks": clk, "calls": calls, "context_at_timed_start": T_timed0,
+            "eq6_ratio": round(eq6_ratio(BLOCK, w.keep, f), 5)}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+ATTR_REPS = 3
+
+
+def run_e2e(args, layers, graph):
+    """Same metric through the public API with host buffers: every step copies
+    its inputs from pinned host memory into the device buffers the captured
+    C-ABI calls read, replays the step, and copies all its outputs back."""
+    import torch
+    f, B, L = layers[0].w.f, layers[0].w.batch, len(layers)
+    dev_in = [[Lc.q, Lc.k, Lc.v, Lc.rq, Lc.rk, Lc.rv] for Lc in layers]
+    dev_out = [[Lc.out, Lc.rout] for Lc in layers]
+    host_in = [[t.cpu().pin_memory() for t in di] for di in dev_in]
+    host_out = [[torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in do] for do in dev_out]
+    h2d = sum(t.numel() * t.element_size() for hi in host_in for t in hi)
+    d2h = sum(t.numel() * t.element_size() for ho in host_out for t in ho)
+    barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps):
+        for di, hi in zip(dev_in, host_in):
+            for d, h in zip(di, hi):
+                d.copy_(h, non_blocking=True)
+        graph.replay()
+        for do, ho in zip(dev_out, host_out):
+            for d, h in zip(do, ho):
+                h.copy_(d, non_blocking=True)
+    e1.record()
+    torch.cuda.synchronize()
+    barrier()
+    secs = max_over_ranks(e0.elapsed_time(e1) / 1e3, layers[0].out.device)
+    _, world, _ = dist_env()
+    return {"value": round(aggregate(B * f * L * args.steps, secs, world), 1), "unit": UNIT,
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "path": "per step: pinned host -> device copies of all inputs, the step's C-ABI calls (captured in a "
+                    "CUDA graph), device -> pinned host copies of every decode and rectify output"}
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--layers", type=int, default=4, help="independent layer caches rotated per decode step")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--oracle-worker", default=None, help=argparse.SUPPRESS)
+    ap.add_argument("--repeats", type=int, default=1, help=argparse.SUPPRESS)
+    args = ap.parse_args()
+    if args.oracle_worker:
+        sample = dict(np.load(args.oracle_worker))
+        print(json.dumps({"seconds": [oracle_period(sample) for _ in range(args.repeats)]}))
+        return
+    if args.warmup < 3 and args.impl == "ours":
+        ap.error("--warmup must be >= 3")
+    w = synth.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        run_reference(args, w)
+    else:
+        run_ours(args, w)
+
+
+if __name__ == "__main__":
+    main()

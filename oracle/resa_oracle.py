@@ -137,6 +137,18 @@ def attend_positions(q: np.ndarray, K: np.ndarray, V: np.ndarray, positions: np.
     return out, lse
 
 
+def attend_prefix(q: np.ndarray, K: np.ndarray, V: np.ndarray, n: int, scale: float):
+    """attend_positions over the contiguous positions [0, n) (views, no gather)."""
+    if n <= 0:
+        g, d = q.shape
+        return np.zeros((g, d)), np.full(g, NEG_INF)
+    logits = (q @ K[:n].T) * scale
+    m = logits.max(axis=1, keepdims=True)
+    e = np.exp(logits - m)
+    den = e.sum(axis=1, keepdims=True)
+    return (e @ V[:n]) / den, (m + np.log(den))[:, 0]
+
+
 def block_positions(blocks: np.ndarray, b: int, T: int) -> np.ndarray:
     """Key positions covered by the given blocks, restricted to [0, T)."""
     if len(blocks) == 0:
@@ -153,7 +165,7 @@ def gbsa_attention(q: np.ndarray, K: np.ndarray, V: np.ndarray, T: int, blocks: 
 
 def dense_attention(q: np.ndarray, K: np.ndarray, V: np.ndarray, T: int, scale: float):
     """Dense attention over positions [0, T) (Eq. 1)."""
-    return attend_positions(q, K, V, np.arange(T), scale)
+    return attend_prefix(q, K, V, T, scale)
 
 
 def split_combine_attention(q, K, V, T, blocks, b, scale, num_splits: int):
@@ -303,7 +315,7 @@ def rectify_attention(q_new: np.ndarray, K: np.ndarray, V: np.ndarray, k_new: np
         Kh = np.concatenate([K[h, :t0], k_new[:, h]], axis=0)   # [T, d]
         Vh = np.concatenate([V[h, :t0], v_new[:, h]], axis=0)
         for i in range(f):
-            o, l = attend_positions(q_new[i, h * g:(h + 1) * g], Kh, Vh, np.arange(t0 + i + 1), scale)
+            o, l = attend_prefix(q_new[i, h * g:(h + 1) * g], Kh, Vh, t0 + i + 1, scale)
             out[i, h * g:(h + 1) * g] = o
             lse[i, h * g:(h + 1) * g] = l
     return out, lse

@@ -1,0 +1,55 @@
+// Internal launcher interface between the C-ABI layer (resa_api.cu) and the
+// kernel translation units. Not part of the public ABI.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "resa.h"
+
+namespace resa {
+
+constexpr int kHeadDimHost = 128;  // supported head_dim
+constexpr int kBlockHost = 16;     // supported block_size (paper's b)
+
+// Plain-old-data view of resa_cache_t handed to kernels by value.
+struct CacheView {
+  int B, Hq, Hkv, g;
+  int num_pages, max_blocks;
+  uint16_t* k_pool;
+  uint16_t* v_pool;
+  const int32_t* page_table;
+  int32_t* seq_lens;
+  uint16_t* summ;
+  int32_t* status;
+};
+
+// Sets cudaFuncAttributeMaxDynamicSharedMemorySize of `func` once per device
+// (kernel-launch paths then make no attribute calls, e.g. under graph capture).
+cudaError_t ensure_smem_attr(const void* func, int bytes, int slot);
+
+// kv_commit.cu
+cudaError_t launch_commit(const CacheView& c, const uint16_t* k_new, const uint16_t* v_new, int n_tokens,
+                          bool overwrite, cudaStream_t st);
+cudaError_t launch_update_summaries(const CacheView& c, int block_begin, int block_end, cudaStream_t st);
+
+// select.cu
+size_t select_smem_bytes(int max_blocks);
+cudaError_t launch_select(const CacheView& c, const uint16_t* q, double keep, int n_min, int n_local,
+                          int32_t* indices, int32_t* counts, int n_cap, float* scores, cudaStream_t st);
+
+// sparse_decode.cu
+cudaError_t launch_sparse_decode(const CacheView& c, const CUtensorMap& tm_k, const CUtensorMap& tm_v,
+                                 const uint16_t* q, const int32_t* indices, const int32_t* counts, int n_cap,
+                                 float sm_scale, int splits, float* o_part, float* lse_part, cudaStream_t st);
+cudaError_t launch_merge(const float* o_part, const float* lse_part, int rows, int splits, uint16_t* out,
+                         float* lse_out, cudaStream_t st);
+
+// rectify.cu
+int rectify_row_groups(int g, int f);
+cudaError_t launch_rectify(const CacheView& c, const CUtensorMap& tm_k, const CUtensorMap& tm_v,
+                           const uint16_t* q_new, const uint16_t* k_new, const uint16_t* v_new, int f,
+                           float sm_scale, int splits, float* o_part, float* lse_part, cudaStream_t st);
+
+}  // namespace resa

@@ -1,0 +1,336 @@
+// Block-sparse split-K flash decoding (Section 2.4; Algorithm 2) and the
+// combine of split partials (Algorithm 2, "Combine").
+//
+// sparse_decode_kernel, grid (splits, KV head, sequence), 4 warps:
+//   * The CTA owns selected blocks [s*per, min(n, (s+1)*per)) of its
+//     (sequence, KV head), per = ceil(n / splits). Warp w takes every 4th of
+//     them, so the group's g <= 8 query heads share every K/V block fetched
+//     (GQA-shared fetch).
+//   * Each warp streams its blocks through a private 3-stage shared-memory
+//     ring: lane 0 issues four bulk-tensor TMA copies per block (K and V, two
+//     64-column halves each, SWIZZLE_128B) that complete on the stage's
+//     mbarrier. Swizzled rows make every ldmatrix below bank-conflict free.
+//   * Per block (16 keys) the warp computes S^T = K * Q^T with 8
+//     m16n8k16 bf16 MMAs (M = 16 keys, N = 8 heads, K = 128 dims), masks keys
+//     at positions >= T, runs the online softmax in the log2 domain, moves
+//     P^T from the accumulator layout to the B-operand layout with movmatrix,
+//     and accumulates O^T += V^T * P^T with 8 more MMAs (V^T via ldmatrix.trans).
+//   * The 4 warps' (m, l, O) are merged through shared memory; the CTA writes
+//     a normalised partial O (fp32) and its log2-sum-exp for each head.
+// merge_kernel, one CTA per output row: LSE-weighted sum of the split partials.
+#include "resa_device.cuh"
+#include "resa_launch.h"
+
+namespace resa {
+namespace {
+
+constexpr int kWarps = 4;
+constexpr int kStages = 3;
+constexpr int kStageBytes = 8192;  // K: 2 x 2 KB halves, V: 2 x 2 KB halves
+constexpr int kRingBytes = kWarps * kStages * kStageBytes;
+constexpr int kDecodeSmem = kRingBytes + 1024 /* alignment slack */ + kWarps * kStages * 8;
+constexpr float kNegInf = -__builtin_huge_valf();
+
+struct DecodeArgs {
+  const uint16_t* q;
+  const int32_t* indices;
+  const int32_t* counts;
+  int n_cap;
+  int splits;
+  float scale_log2;
+  float* o_part;    // [B][Hq][splits][128]
+  float* lse_part;  // [B][Hq][splits], log2 domain
+};
+
+__device__ __forceinline__ float safe_base(float m) { return m == kNegInf ? 0.f : m; }
+
+__global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid_constant__ CUtensorMap tm_k,
+                                                                    const __grid_constant__ CUtensorMap tm_v,
+                                                                    CacheView c, DecodeArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kRingBytes);
+  __shared__ float wm[kWarps][8], wl[kWarps][8];
+
+  const int s = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int T = c.seq_lens[b];
+  int n = a.counts[b * c.Hkv + h];
+  if (T < 0 || T > c.max_blocks * kBlock) {
+    if (threadIdx.x == 0 && s == 0) record_error(c.status, RESA_DEV_SEQ_LEN_RANGE, b);
+    n = 0;
+  } else if (n < 0 || n > a.n_cap) {
+    if (threadIdx.x == 0 && s == 0) record_error(c.status, RESA_DEV_BAD_INDEX, b * c.Hkv + h);
+    n = 0;
+  }
+  const int M = (max(T, 0) + kBlock - 1) / kBlock;
+  const int per = (n + a.splits - 1) / a.splits;
+  const int j0 = s * per;
+  const int nj = max(0, min(n, j0 + per) - j0);
+  const int cnt = nj > warp ? (nj - warp + kWarps - 1) / kWarps : 0;
+  const int32_t* idx = a.indices + static_cast<size_t>(b * c.Hkv + h) * a.n_cap + j0 + warp;
+
+  const uint32_t ring = smem_u32(smem) + warp * kStages * kStageBytes;
+  const uint32_t bar0 = smem_u32(bars + warp * kStages);
+  if (lane == 0) {
+    for (int st = 0; st < kStages; ++st) mbar_init(bar0 + 8 * st, 1);
+    fence_mbar_init();
+  }
+  __syncwarp();
+
+  // Page of the it-th block of this warp, or -1 if the block id or its page
+  // is out of range (the block is then treated as fully masked).
+  auto page_of = [&](int it, int& blk) -> int {
+    blk = idx[it * kWarps];
+    if (blk < 0 || blk >= M) return -1;
+    const int page = c.page_table[static_cast<size_t>(b) * c.max_blocks + blk];
+    return (page >= 0 && page < c.num_pages) ? page : -2;
+  };
+  auto issue = [&](int it, int st) {  // lane 0 only
+    int blk;
+    const int page = page_of(it, blk);
+    const uint32_t bar = bar0 + 8 * st;
+    if (page < 0) {
+      record_error(c.status, page == -1 ? RESA_DEV_BAD_INDEX : RESA_DEV_PAGE_RANGE, b * c.Hkv + h);
+      mbar_arrive(bar);  // completes the phase with no data
+      return;
+    }
+    const int row = (page * c.Hkv + h) * kBlock;
+    const uint32_t dst = ring + st * kStageBytes;
+    mbar_arrive_expect_tx(bar, kStageBytes);
+    tma_load_2d(dst, &tm_k, bar, 0, row);
+    tma_load_2d(dst + 2048, &tm_k, bar, 64, row);
+    tma_load_2d(dst + 4096, &tm_v, bar, 0, row);
+    tma_load_2d(dst + 6144, &tm_v, bar, 64, row);
+  };
+
+  // Q^T as the B operand: lane holds head lane/4, dims 16ks + 2(lane%4) (+1, +8, +9).
+  uint32_t qb[8][2];
+  {
+    const int qh = lane >> 2;
+    const bool ok = qh < c.g;
+    const uint16_t* qr = a.q + (static_cast<size_t>(b) * c.Hq + h * c.g + (ok ? qh : 0)) * kHeadDim;
+#pragma unroll
+    for (int ks = 0; ks < 8; ++ks) {
+      const int d0 = 16 * ks + 2 * (lane & 3);
+      qb[ks][0] = ok ? *reinterpret_cast<const uint32_t*>(qr + d0) : 0u;
+      qb[ks][1] = ok ? *reinterpret_cast<const uint32_t*>(qr + d0 + 8) : 0u;
+    }
+  }
+
+  int issued = 0;
+  if (lane == 0) {
+    prefetch_tmap(&tm_k);
+    prefetch_tmap(&tm_v);
+    for (; issued < min(kStages, cnt); ++issued) issue(issued, issued);
+  }
+  issued = __shfl_sync(0xffffffffu, issued, 0);
+
+  float m0 = kNegInf, m1 = kNegInf, l0 = 0.f, l1 = 0.f;
+  float acc[8][4];
+#pragma unroll
+  for (int mt = 0; mt < 8; ++mt) acc[mt][0] = acc[mt][1] = acc[mt][2] = acc[mt][3] = 0.f;
+
+  int it = 0;
+  for (; it < cnt; ++it) {
+    const int st = it % kStages;
+    const uint32_t par = (it / kStages) & 1;
+    const uint32_t bar = bar0 + 8 * st;
+    int ok = 1;
+    if (lane == 0) ok = mbar_wait_bounded(bar, par) ? 1 : 0;
+    ok = __shfl_sync(0xffffffffu, ok, 0);
+    if (!ok) {
+      if (lane == 0) record_error(c.status, RESA_DEV_WAIT_TIMEOUT, b * c.Hkv + h);
+      break;
+    }
+    mbar_try_wait(bar, par);  // acquire for every lane (the phase has completed)
+    int blk;
+    const int page = page_of(it, blk);
+    const int valid = page < 0 ? 0 : min(kBlock, T - blk * kBlock);
+    const uint32_t kb = ring + st * kStageBytes, vb = kb + 4096;
+    if (valid < kBlock) {  // rows past the end (or an invalid block) may hold garbage: zero V
+      uint8_t* v = smem + (kb - smem_u32(smem)) + 4096;
+      for (int e = lane; e < (kBlock - valid) * 16; e += 32) {
+        const int r = valid + (e >> 4), half = (e >> 3) & 1, chunk = e & 7;
+        *reinterpret_cast<uint4*>(v + half * 2048 + r * 128 + chunk * 16) = make_uint4(0, 0, 0, 0);
+      }
+      __syncwarp();
+    }
+    // S^T = K * Q^T
+    float sc[4] = {0.f, 0.f, 0.f, 0.f};
+    {
+      const int key = (lane & 7) + ((lane >> 3) & 1) * 8;
+#pragma unroll
+      for (int ks = 0; ks < 8; ++ks) {
+        const int chunk = 2 * ks + (lane >> 4);
+        uint32_t a0, a1, a2, a3;
+        ldsm_x4(kb + (chunk >> 3) * 2048 + sw128(key, chunk & 7), a0, a1, a2, a3);
+        mma_bf16_16816(sc, a0, a1, a2, a3, qb[ks][0], qb[ks][1]);
+      }
+    }
+    const int k0 = lane >> 2;
+    float s0 = (k0 < valid) ? sc[0] * a.scale_log2 : kNegInf;
+    float s1 = (k0 < valid) ? sc[1] * a.scale_log2 : kNegInf;
+    float s2 = (k0 + 8 < valid) ? sc[2] * a.scale_log2 : kNegInf;
+    float s3 = (k0 + 8 < valid) ? sc[3] * a.scale_log2 : kNegInf;
+    float bm0 = fmaxf(s0, s2), bm1 = fmaxf(s1, s3);
+#pragma unroll
+    for (int o = 4; o < 32; o <<= 1) {
+      bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, o));
+      bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, o));
+    }
+    const float n0 = fmaxf(m0, bm0), n1 = fmaxf(m1, bm1);
+    const float base0 = safe_base(n0), base1 = safe_base(n1);
+    const float al0 = exp2f(m0 - base0), al1 = exp2f(m1 - base1);
+    const uint32_t x0 = pack_bf16x2(exp2f(s0 - base0), exp2f(s1 - base1));
+    const uint32_t x1 = pack_bf16x2(exp2f(s2 - base0), exp2f(s3 - base1));
+    l0 = l0 * al0 + bf16_lo(x0) + bf16_lo(x1);
+    l1 = l1 * al1 + bf16_hi(x0) + bf16_hi(x1);
+    m0 = n0;
+    m1 = n1;
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt) {
+      acc[mt][0] *= al0;
+      acc[mt][1] *= al1;
+      acc[mt][2] *= al0;
+      acc[mt][3] *= al1;
+    }
+    const uint32_t pb0 = movmatrix_t(x0), pb1 = movmatrix_t(x1);
+    // O^T += V^T * P^T
+    {
+      const int j = lane >> 3;
+      const int key = (lane & 7) + (j >> 1) * 8;
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) {
+        const int chunk = 2 * mt + (j & 1);
+        uint32_t a0, a1, a2, a3;
+        ldsm_x4_t(vb + (chunk >> 3) * 2048 + sw128(key, chunk & 7), a0, a1, a2, a3);
+        mma_bf16_16816(acc[mt], a0, a1, a2, a3, pb0, pb1);
+      }
+    }
+    __syncwarp();
+    if (issued < cnt) {
+      if (lane == 0) {
+        fence_proxy_async_smem();
+        issue(issued, st);
+      }
+      ++issued;
+    }
+  }
+  if (it < cnt && lane == 0) {  // timed out: let copies already in flight land before leaving
+    for (int k = it; k < issued; ++k) mbar_wait_bounded(bar0 + 8 * (k % kStages), (k / kStages) & 1);
+  }
+
+  // ---- merge the 4 warps' softmax states ----
+#pragma unroll
+  for (int o = 4; o < 32; o <<= 1) {
+    l0 += __shfl_xor_sync(0xffffffffu, l0, o);
+    l1 += __shfl_xor_sync(0xffffffffu, l1, o);
+  }
+  if (lane < 4) {
+    wm[warp][2 * lane] = m0;
+    wm[warp][2 * lane + 1] = m1;
+    wl[warp][2 * lane] = l0;
+    wl[warp][2 * lane + 1] = l1;
+  }
+  __syncthreads();
+  const int hA = 2 * (lane & 3), hB = hA + 1;
+  float MA = kNegInf, MB = kNegInf;
+#pragma unroll
+  for (int w = 0; w < kWarps; ++w) {
+    MA = fmaxf(MA, wm[w][hA]);
+    MB = fmaxf(MB, wm[w][hB]);
+  }
+  float LA = 0.f, LB = 0.f;
+#pragma unroll
+  for (int w = 0; w < kWarps; ++w) {
+    LA += wl[w][hA] * exp2f(wm[w][hA] - safe_base(MA));
+    LB += wl[w][hB] * exp2f(wm[w][hB] - safe_base(MB));
+  }
+  const float fA = LA > 0.f ? exp2f(m0 - safe_base(MA)) / LA : 0.f;
+  const float fB = LB > 0.f ? exp2f(m1 - safe_base(MB)) / LB : 0.f;
+  float* red = reinterpret_cast<float*>(smem);  // [warp][8 heads][128] fp32, reuses the ring
+#pragma unroll
+  for (int mt = 0; mt < 8; ++mt) {
+    const int dA = 16 * mt + (lane >> 2), dB = dA + 8;
+    red[(warp * 8 + hA) * kHeadDim + dA] = acc[mt][0] * fA;
+    red[(warp * 8 + hB) * kHeadDim + dA] = acc[mt][1] * fB;
+    red[(warp * 8 + hA) * kHeadDim + dB] = acc[mt][2] * fA;
+    red[(warp * 8 + hB) * kHeadDim + dB] = acc[mt][3] * fB;
+  }
+  __syncthreads();
+  const int t = threadIdx.x;  // one output dim per thread
+  for (int hh = 0; hh < c.g; ++hh) {
+    float v = 0.f;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) v += red[(w * 8 + hh) * kHeadDim + t];
+    const size_t row = static_cast<size_t>(b) * c.Hq + h * c.g + hh;
+    a.o_part[(row * a.splits + s) * kHeadDim + t] = v;
+  }
+  if (t < c.g) {
+    float Mt = kNegInf;
+    for (int w = 0; w < kWarps; ++w) Mt = fmaxf(Mt, wm[w][t]);
+    float Lt = 0.f;
+    for (int w = 0; w < kWarps; ++w) Lt += wl[w][t] * exp2f(wm[w][t] - safe_base(Mt));
+    const size_t row = static_cast<size_t>(b) * c.Hq + h * c.g + t;
+    a.lse_part[row * a.splits + s] = Lt > 0.f ? Mt + log2f(Lt) : kNegInf;
+  }
+}
+
+__global__ void __launch_bounds__(128) merge_kernel(const float* __restrict__ o_part,
+                                                    const float* __restrict__ lse_part, int splits,
+                                                    uint16_t* __restrict__ out, float* __restrict__ lse_out) {
+  extern __shared__ float w[];
+  __shared__ float sh_m, sh_l;
+  const size_t row = blockIdx.x;
+  const int t = threadIdx.x;
+  const float* lp = lse_part + row * splits;
+  if (t < 32) {
+    float m = kNegInf;
+    for (int s = t; s < splits; s += 32) m = fmaxf(m, lp[s]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    if (t == 0) sh_m = m;
+  }
+  __syncthreads();
+  const float M = sh_m;
+  for (int s = t; s < splits; s += 128) w[s] = (lp[s] == kNegInf) ? 0.f : exp2f(lp[s] - M);
+  __syncthreads();
+  if (t < 32) {
+    float l = 0.f;
+    for (int s = t; s < splits; s += 32) l += w[s];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+    if (t == 0) sh_l = l;
+  }
+  __syncthreads();
+  const float L = sh_l;
+  const float inv = L > 0.f ? 1.f / L : 0.f;
+  const float* op = o_part + row * splits * kHeadDim + t;
+  float v = 0.f;
+  for (int s = 0; s < splits; ++s) v += w[s] * op[static_cast<size_t>(s) * kHeadDim];
+  const __nv_bfloat16 r = __float2bfloat16_rn(v * inv);
+  out[row * kHeadDim + t] = *reinterpret_cast<const uint16_t*>(&r);
+  if (lse_out != nullptr && t == 0) lse_out[row] = L > 0.f ? (M + log2f(L)) * 0.69314718055994530942f : kNegInf;
+}
+
+}  // namespace
+
+cudaError_t launch_sparse_decode(const CacheView& c, const CUtensorMap& tm_k, const CUtensorMap& tm_v,
+                                 const uint16_t* q, const int32_t* indices, const int32_t* counts, int n_cap,
+                                 float sm_scale, int splits, float* o_part, float* lse_part, cudaStream_t st) {
+  cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(sparse_decode_kernel), kDecodeSmem, 0);
+  if (e != cudaSuccess) return e;
+  DecodeArgs a{q, indices, counts, n_cap, splits, sm_scale * 1.44269504088896340736f, o_part, lse_part};
+  sparse_decode_kernel<<<dim3(splits, c.Hkv, c.B), kWarps * 32, kDecodeSmem, st>>>(tm_k, tm_v, c, a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_merge(const float* o_part, const float* lse_part, int rows, int splits, uint16_t* out,
+                         float* lse_out, cudaStream_t st) {
+  if (rows == 0) return cudaSuccess;
+  merge_kernel<<<rows, 128, splits * sizeof(float), st>>>(o_part, lse_part, splits, out, lse_out);
+  return cudaGetLastError();
+}
+
+}  // namespace resa

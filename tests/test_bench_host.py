@@ -1,0 +1,70 @@
+"""Host-side logic of bench.py (CPU only): the algorithmic byte model against
+Eq. 6, and the multi-rank aggregation over a world_size-2 gloo group."""
+import math
+import os
+
+import pytest
+import torch
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+import bench
+
+
+def test_step_bytes_follow_eq6():
+    """Per decode step: summaries (1/b of the KV cache) + selected KV (keep) +
+    amortised rectification (1/f) ~= Eq. 6 times the KV bytes. The small
+    extra terms (fp32 scores, queries, outputs, partial last block) stay
+    within 3%."""
+    B, Hq, Hkv, T, f = 8, 28, 4, 32768, 32
+    kv = B * Hkv * T * 2 * 128 * 2
+    M = T // 16
+    per_step = (bench.select_bytes(B, Hq, Hkv, T, 0.1, 0, 1) + bench.decode_bytes(B, Hq, Hkv, T, 0.1, 0, 1)
+                + bench.rectify_bytes(B, Hq, Hkv, T, f) / f)
+    ratio = per_step / kv
+    assert math.isclose(bench.eq6_ratio(16, 0.1, 32), 0.19375)
+    assert abs(ratio - bench.eq6_ratio(16, 0.1, 32)) / 0.19375 < 0.03
+    assert bench.budget(M, 0.1, 128, 1) == 205
+
+
+def test_decode_bytes_count_valid_tokens_of_partial_block():
+    # T = 33: M = 3 blocks, all kept; 33 tokens attended
+    assert bench.decode_bytes(1, 1, 1, 33, 1.0, 0, 1) == 33 * 512 + 2 * 256
+
+
+def test_rectify_flops_causal_count():
+    # f = 2 rows at T = 10: row 0 sees 9 keys, row 1 sees 10
+    assert bench.rectify_flops(1, 1, 10, 2) == 4 * 128 * (9 + 10)
+
+
+def _rank_main(rank, world, port, q):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(world),
+                      LOCAL_RANK=str(rank))
+    r, w = bench.init_dist("gloo")
+    bench.barrier()
+    secs = 1.0 + rank                      # rank 1 is the slow one
+    m = bench.max_over_ranks(secs)
+    q.put((r, w, m, bench.aggregate(100.0, m, w)))
+    dist.destroy_process_group()
+
+
+def test_two_rank_gloo_aggregation():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = 29500 + (os.getpid() % 1000)
+    procs = [ctx.Process(target=_rank_main, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    res = sorted(q.get(timeout=120) for _ in procs)
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    for r, (rank, world, m, value) in enumerate(res):
+        assert rank == r and world == 2
+        assert m == pytest.approx(2.0)          # max over ranks
+        assert value == pytest.approx(100.0 * 2 / 2.0)
+
+
+def test_single_process_helpers_are_identity():
+    assert bench.max_over_ranks(3.5) == 3.5
+    assert bench.aggregate(10.0, 2.0, 1) == 5.0

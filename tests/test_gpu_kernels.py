@@ -1,0 +1,300 @@
+"""Per-call parity of the CUDA path (through the C ABI) against the fp64 oracle
+on seeded inputs: cache commit / summaries (bit-exact), block selection
+(exact up to the near-tie rule), sparse decode and rectification (2e-2
+max-abs, 1e-3 mean-abs), plus device-side error reporting."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2506_04108_gb300 import resa, synth
+from tests import gpu_harness as H
+
+pytestmark = pytest.mark.gpu
+
+
+def seq_inputs(seed, B, Hkv, lens, d=128, k_scale=1.0):
+    g = synth.rng(seed)
+    Ks = [synth.normal_bf16(g, (Hkv, T, d), k_scale) for T in lens]
+    Vs = [synth.normal_bf16(g, (Hkv, T, d)) for T in lens]
+    return Ks, Vs
+
+
+# ---------------------------------------------------------------- Eq. 3 ---
+@pytest.mark.parametrize("lens", [[16], [1, 17, 100, 333], [4096, 4095]])
+def test_update_summaries_bit_exact(lens):
+    Hkv = 2
+    Ks, Vs = seq_inputs(1, len(lens), Hkv, lens)
+    maxb = (max(lens) + 15) // 16 + 3
+    cache = H.make_cache(Ks, Vs, Hkv * 4, maxb, zero_pools=False)
+    summ = H.host_f64(cache.summaries)          # [B, Hkv, maxb, 2, d]
+    for b, T in enumerate(lens):
+        M = (T + 15) // 16
+        for h in range(Hkv):
+            mn, mx = O.block_summaries(O.widen_bf16(Ks[b][h]), 16)
+            assert np.array_equal(summ[b, h, :M, 0], mn)
+            assert np.array_equal(summ[b, h, :M, 1], mx)
+    assert resa.resa_read_device_error(cache.struct) == (0, 0)
+
+
+def test_update_summaries_range_only_touches_range():
+    Ks, Vs = seq_inputs(2, 1, 1, [200])
+    cache = H.make_cache(Ks, Vs, 2, 16)
+    cache.summaries.zero_()
+    resa.resa_update_summaries(cache.struct, 3, 7)
+    s = H.host_f64(cache.summaries)[0, 0]
+    mn, mx = O.block_summaries(O.widen_bf16(Ks[0][0]), 16)
+    assert np.all(s[:3] == 0) and np.all(s[7:] == 0)
+    assert np.array_equal(s[3:7, 0], mn[3:7]) and np.array_equal(s[3:7, 1], mx[3:7])
+
+
+@pytest.mark.parametrize("lens,n_new", [([30, 16, 1], 1), ([30, 47, 64], 5), ([0, 15, 16], 20)])
+def test_commit_append_matches_oracle(lens, n_new):
+    Hkv, d = 2, 128
+    Ks, Vs = seq_inputs(3, len(lens), Hkv, lens)
+    maxb = 8
+    cache = H.make_cache(Ks, Vs, 4, maxb)
+    g = synth.rng(33)
+    kn = synth.normal_bf16(g, (len(lens), n_new, Hkv, d))
+    vn = synth.normal_bf16(g, (len(lens), n_new, Hkv, d))
+    resa.resa_commit_kv(cache.struct, H.dev_bf16(kn), H.dev_bf16(vn), n_new, False)
+    assert resa.resa_read_device_error(cache.struct) == (0, 0)
+    summ = H.host_f64(cache.summaries)
+    for b, T in enumerate(lens):
+        st = H.oracle_state(Ks[b], Vs[b], maxb * 16)
+        for t in range(n_new):
+            st.append(O.widen_bf16(kn[b, t]), O.widen_bf16(vn[b, t]))
+        assert int(cache.seq_lens[b]) == T + n_new
+        K, V = H.logical_kv(cache, b)
+        assert np.array_equal(O.widen_bf16(K), st.K[:, :st.T]) and np.array_equal(O.widen_bf16(V), st.V[:, :st.T])
+        M = st.num_blocks
+        assert np.array_equal(summ[b, :, :M, 0], st.kmin[:, :M]) and np.array_equal(summ[b, :, :M, 1], st.kmax[:, :M])
+
+
+@pytest.mark.parametrize("lens,f", [([64, 100], 8), ([37, 333], 32), ([64, 200], 64), ([16, 17], 16)])
+def test_commit_overwrite_matches_oracle(lens, f):
+    Hkv, d = 4, 128
+    Ks, Vs = seq_inputs(4, len(lens), Hkv, lens)
+    maxb = 24
+    cache = H.make_cache(Ks, Vs, 28, maxb)
+    g = synth.rng(44)
+    kn = synth.normal_bf16(g, (len(lens), f, Hkv, d))
+    vn = synth.normal_bf16(g, (len(lens), f, Hkv, d))
+    resa.resa_commit_kv(cache.struct, H.dev_bf16(kn), H.dev_bf16(vn), f, True)
+    assert resa.resa_read_device_error(cache.struct) == (0, 0)
+    summ = H.host_f64(cache.summaries)
+    for b, T in enumerate(lens):
+        st = H.oracle_state(Ks[b], Vs[b], maxb * 16)
+        st.overwrite_tail(O.widen_bf16(kn[b]), O.widen_bf16(vn[b]))
+        assert int(cache.seq_lens[b]) == T
+        K, V = H.logical_kv(cache, b)
+        assert np.array_equal(O.widen_bf16(K), st.K[:, :T]) and np.array_equal(O.widen_bf16(V), st.V[:, :T])
+        M = st.num_blocks
+        assert np.array_equal(summ[b, :, :M, 0], st.kmin[:, :M]) and np.array_equal(summ[b, :, :M, 1], st.kmax[:, :M])
+
+
+# ---------------------------------------------------------- Eq. 4 / 5 -----
+def run_select(cache, q_bits, p, n_cap):
+    B, Hkv = cache.batch, cache.Hkv
+    idx = torch.empty((B, Hkv, n_cap), dtype=torch.int32, device="cuda")
+    cnt = torch.empty((B, Hkv), dtype=torch.int32, device="cuda")
+    ws, nb = H.workspace(cache, n_cap)
+    resa.resa_select_blocks(cache.struct, H.dev_bf16(q_bits), p, idx, cnt, n_cap, ws, nb)
+    return idx.cpu().numpy(), cnt.cpu().numpy()
+
+
+@pytest.mark.parametrize("g,Hkv,lens,keep,n_min,n_local", [
+    (4, 2, [4100], 0.1, 16, 4),            # the 4K workload shape
+    (7, 4, [1000, 2053, 37, 16], 0.1, 8, 1),
+    (1, 1, [513], 0.25, 0, 0),
+    (8, 1, [300, 5000], 0.05, 3, 2),
+    (7, 4, [100, 80], 0.5, 16, 1),         # M <= n: every block selected
+    (2, 2, [160], 0.0, 0, 12),             # n_local >= n
+])
+def test_select_matches_oracle(g, Hkv, lens, keep, n_min, n_local):
+    Ks, Vs = seq_inputs(5 + len(lens), len(lens), Hkv, lens)
+    maxb = max((T + 15) // 16 for T in lens) + 4
+    cache = H.make_cache(Ks, Vs, g * Hkv, maxb)
+    gq = synth.rng(55)
+    q = synth.normal_bf16(gq, (len(lens), g * Hkv, 128))
+    p = resa.params(keep, n_min, n_local)
+    n_cap = resa.resa_max_selected(cache.struct, p) + 3
+    idx, cnt = run_select(cache, q, p, n_cap)
+    assert resa.resa_read_device_error(cache.struct) == (0, 0)
+    for b, T in enumerate(lens):
+        st = H.oracle_state(Ks[b], Vs[b], maxb * 16)
+        for h in range(Hkv):
+            sel, scores, n = O.select_for_group(st, h, O.widen_bf16(q[b, h * g:(h + 1) * g]),
+                                                O.ResaParams(keep, n_min, n_local))
+            assert cnt[b, h] == n
+            assert np.all(idx[b, h, n:] == -1)
+            H.check_selection(idx[b, h, :n], scores, n, n_local)
+
+
+def test_select_ties_go_to_lower_index():
+    """Identical blocks give identical scores; the lower ids must win."""
+    Hkv, g, T = 1, 4, 16 * 40
+    blk = synth.normal_bf16(synth.rng(6), (Hkv, 16, 128))
+    K = np.tile(blk, (1, 40, 1))
+    V = synth.normal_bf16(synth.rng(7), (Hkv, T, 128))
+    cache = H.make_cache([K], [V], g, 44)
+    q = synth.normal_bf16(synth.rng(8), (1, g, 128))
+    p = resa.params(0.1, 0, 1)
+    idx, cnt = run_select(cache, q, p, 16)
+    assert cnt[0, 0] == 4
+    assert idx[0, 0, :4].tolist() == [0, 1, 2, 39]
+
+
+def test_select_budget_over_cap_is_reported_and_clamped():
+    Ks, Vs = seq_inputs(9, 1, 1, [1600])
+    cache = H.make_cache(Ks, Vs, 2, 110)
+    q = synth.normal_bf16(synth.rng(9), (1, 2, 128))
+    p = resa.params(0.1, 0, 1)
+    idx, cnt = run_select(cache, q, p, 5)               # n = 10 > n_cap = 5
+    code, _ = resa.resa_read_device_error(cache.struct)
+    assert code == 3 and cnt[0, 0] == 5
+    assert len(set(idx[0, 0].tolist())) == 5
+
+
+# ------------------------------------------------------ Eq. 2 / Alg. 2 ----
+def run_decode(cache, q_bits, sel_rows, n_cap, p, splits):
+    """sel_rows[b][h] = block ids (any order)."""
+    B, Hkv, Hq = cache.batch, cache.Hkv, cache.Hq
+    idx = np.full((B, Hkv, n_cap), -1, dtype=np.int32)
+    cnt = np.zeros((B, Hkv), dtype=np.int32)
+    for b in range(B):
+        for h in range(Hkv):
+            s = np.asarray(sel_rows[b][h], dtype=np.int32)
+            idx[b, h, :len(s)] = s
+            cnt[b, h] = len(s)
+    out = torch.empty((B, Hq, 128), dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty((B, Hq), dtype=torch.float32, device="cuda")
+    ws, nb = H.workspace(cache, n_cap, splits)
+    resa.resa_sparse_decode(cache.struct, H.dev_bf16(q_bits), torch.from_numpy(idx).cuda(),
+                            torch.from_numpy(cnt).cuda(), n_cap, p, out, lse, splits, ws, nb)
+    return H.host_f64(out), lse.cpu().numpy().astype(np.float64)
+
+
+@pytest.mark.parametrize("g,Hkv,lens,nsel,splits", [
+    (4, 2, [4100], 26, 0), (7, 4, [2053, 999], 40, 0), (7, 4, [2053, 999], 40, 1), (7, 4, [2053], 40, 7),
+    (8, 1, [33], 3, 64), (1, 2, [500], 1, 0), (7, 1, [16 * 300 + 5], 300, 0), (2, 1, [17], 2, 3),
+])
+def test_sparse_decode_matches_oracle(g, Hkv, lens, nsel, splits):
+    Ks, Vs = seq_inputs(10 + g, len(lens), Hkv, lens)
+    maxb = max((T + 15) // 16 for T in lens) + 2
+    cache = H.make_cache(Ks, Vs, g * Hkv, maxb)
+    gr = synth.rng(77)
+    q = synth.normal_bf16(gr, (len(lens), g * Hkv, 128))
+    sel = []
+    for b, T in enumerate(lens):
+        M = (T + 15) // 16
+        rows = []
+        for h in range(Hkv):
+            s = np.sort(gr.choice(M, size=min(nsel, M), replace=False))
+            if M - 1 not in s:               # always include the partial last block
+                s[-1] = M - 1
+                s = np.unique(s)
+            rows.append(s)
+        sel.append(rows)
+    n_cap = max(len(r) for rows in sel for r in rows) + 1
+    p = resa.params(0.1, 0, 0)
+    out, lse = run_decode(cache, q, sel, n_cap, p, splits)
+    assert resa.resa_read_device_error(cache.struct) == (0, 0)
+    sc = 1 / math.sqrt(128)
+    for b, T in enumerate(lens):
+        Kf, Vf = O.widen_bf16(Ks[b]), O.widen_bf16(Vs[b])
+        for h in range(Hkv):
+            o, l = O.gbsa_attention(O.widen_bf16(q[b, h * g:(h + 1) * g]), Kf[h], Vf[h], T, sel[b][h], 16, sc)
+            H.check_outputs(out[b, h * g:(h + 1) * g], o, f"b{b} h{h}")
+            assert np.allclose(lse[b, h * g:(h + 1) * g], l, atol=2e-3, rtol=0)
+
+
+def test_sparse_decode_all_blocks_equals_dense():
+    g, Hkv, T = 7, 1, 16 * 64 - 3
+    Ks, Vs = seq_inputs(21, 1, Hkv, [T])
+    cache = H.make_cache(Ks, Vs, g, 64)
+    q = synth.normal_bf16(synth.rng(22), (1, g, 128))
+    out, _ = run_decode(cache, q, [[np.arange(64)]], 64, resa.params(1.0, 0, 0), 0)
+    o, _ = O.dense_attention(O.widen_bf16(q[0]), O.widen_bf16(Ks[0][0]), O.widen_bf16(Vs[0][0]), T,
+                             1 / math.sqrt(128))
+    H.check_outputs(out[0], o, "dense")
+
+
+def test_sparse_decode_empty_selection_gives_zero_and_neg_inf():
+    Ks, Vs = seq_inputs(23, 1, 1, [64])
+    cache = H.make_cache(Ks, Vs, 4, 4)
+    q = synth.normal_bf16(synth.rng(24), (1, 4, 128))
+    out, lse = run_decode(cache, q, [[np.zeros(0, dtype=np.int32)]], 4, resa.params(0.1, 0, 0), 0)
+    assert np.all(out == 0) and np.all(np.isneginf(lse))
+
+
+def test_sparse_decode_bad_block_id_is_reported_not_faulted():
+    Ks, Vs = seq_inputs(25, 1, 1, [64])
+    cache = H.make_cache(Ks, Vs, 4, 4)
+    q = synth.normal_bf16(synth.rng(26), (1, 4, 128))
+    out, _ = run_decode(cache, q, [[np.array([0, 7])]], 4, resa.params(0.1, 0, 0), 1)   # block 7 >= M = 4
+    code, _ = resa.resa_read_device_error(cache.struct)
+    assert code == 5
+    o, _ = O.gbsa_attention(O.widen_bf16(q[0]), O.widen_bf16(Ks[0][0]), O.widen_bf16(Vs[0][0]), 64, [0], 16,
+                            1 / math.sqrt(128))
+    H.check_outputs(out[0], o, "bad id treated as masked")
+
+
+# ------------------------------------------------------- rectification ----
+@pytest.mark.parametrize("g,Hkv,lens,f", [
+    (4, 2, [4100], 8), (7, 4, [2053, 640], 32), (7, 1, [1000], 16), (7, 1, [777], 64), (8, 2, [64], 64),
+    (1, 1, [300], 8), (7, 2, [32], 32),
+])
+def test_rectify_matches_oracle(g, Hkv, lens, f):
+    Ks, Vs = seq_inputs(30 + f, len(lens), Hkv, lens)
+    maxb = max((T + 15) // 16 for T in lens) + 2
+    cache = H.make_cache(Ks, Vs, g * Hkv, maxb)
+    gr = synth.rng(88)
+    B = len(lens)
+    qn = synth.normal_bf16(gr, (B, f, g * Hkv, 128))
+    kn = synth.normal_bf16(gr, (B, f, Hkv, 128))
+    vn = synth.normal_bf16(gr, (B, f, Hkv, 128))
+    out = torch.empty((B, f, g * Hkv, 128), dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty((B, f, g * Hkv), dtype=torch.float32, device="cuda")
+    ws, nb = H.workspace(cache, 8, 0, f)
+    p = resa.params(0.1, 16, 1)
+    resa.resa_rectify_attention(cache.struct, H.dev_bf16(qn), H.dev_bf16(kn), H.dev_bf16(vn), f, p, out, lse, ws, nb)
+    assert resa.resa_read_device_error(cache.struct) == (0, 0)
+    out, lse = H.host_f64(out), lse.cpu().numpy()
+    for b, T in enumerate(lens):
+        o, l = O.rectify_attention(O.widen_bf16(qn[b]), O.widen_bf16(Ks[b]), O.widen_bf16(Vs[b]),
+                                   O.widen_bf16(kn[b]), O.widen_bf16(vn[b]), T, 1 / math.sqrt(128))
+        H.check_outputs(out[b], o, f"rectify b{b}")
+        assert np.allclose(lse[b], l, atol=2e-3, rtol=0)
+
+
+def test_rectify_too_short_sequence_is_reported():
+    Ks, Vs = seq_inputs(40, 1, 1, [8])
+    cache = H.make_cache(Ks, Vs, 4, 4)
+    f = 16
+    z = torch.zeros((1, f, 4, 128), dtype=torch.bfloat16, device="cuda")
+    zk = torch.zeros((1, f, 1, 128), dtype=torch.bfloat16, device="cuda")
+    out = torch.empty_like(z)
+    ws, nb = H.workspace(cache, 4, 0, f)
+    resa.resa_rectify_attention(cache.struct, z, zk, zk, f, resa.params(0.1, 0, 0), out, None, ws, nb)
+    assert resa.resa_read_device_error(cache.struct)[0] == 1
+
+
+def test_commit_beyond_capacity_is_reported_and_skipped():
+    Ks, Vs = seq_inputs(41, 1, 1, [60])
+    cache = H.make_cache(Ks, Vs, 2, 4)            # capacity 64
+    kn = torch.zeros((1, 5, 1, 128), dtype=torch.bfloat16, device="cuda")
+    resa.resa_commit_kv(cache.struct, kn, kn, 5, False)
+    assert resa.resa_read_device_error(cache.struct)[0] == 1
+    assert int(cache.seq_lens[0]) == 60
+
+
+def test_bad_page_table_entry_is_reported():
+    Ks, Vs = seq_inputs(42, 1, 1, [40])
+    cache = H.make_cache(Ks, Vs, 2, 4)
+    cache.page_table[0, 2] = 10 ** 6
+    kn = torch.zeros((1, 1, 1, 128), dtype=torch.bfloat16, device="cuda")
+    resa.resa_commit_kv(cache.struct, kn, kn, 1, False)
+    assert resa.resa_read_device_error(cache.struct)[0] == 2
