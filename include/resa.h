@@ -238,6 +238,33 @@ resa_status_t resa_rectify_attention(const resa_cache_t* cache, const void* q_ne
                                      float* lse, void* workspace, size_t workspace_bytes, void* stream);
 
 /*
+ * resa_sparse_decode without a caller workspace. The paper has no counterpart:
+ * this entry point exists for callers that cannot allocate device memory --
+ * for example a plugin inside a host framework that owns all device memory
+ * and hands its plugins no allocator, or code on a latency-critical path
+ * where a device allocation (which may synchronise the device) is not
+ * allowed. It computes exactly what resa_sparse_decode computes, with the
+ * same arguments minus the workspace; the split partials live instead in one
+ * library-owned static device buffer of RESA_STATIC_SCRATCH_BYTES, which
+ * every GPU that loads the library holds until the process exits.
+ *   - It calls no cudaMalloc / cudaFree or any allocating routine.
+ *   - Calls whose partials need more than RESA_STATIC_SCRATCH_BYTES
+ *     (batch * num_q_heads * splits * (head_dim + 1) * 4 bytes, each part
+ *     rounded up to 256 bytes) return RESA_ERR_WORKSPACE and launch nothing.
+ *   - The first call on a device looks up the buffer's device address (with
+ *     that device current) and caches it; make that first call before any
+ *     stream capture on that device.
+ *   - All calls share the one buffer, and it keeps the last call's contents
+ *     (nothing in it needs to start at zero: every call overwrites every
+ *     partial it reads). Calls that overlap on the GPU (e.g. on two streams
+ *     without ordering) race on the buffer and give undefined results.
+ */
+#define RESA_STATIC_SCRATCH_BYTES (4u * 1024u * 1024u)
+resa_status_t resa_sparse_decode_static(const resa_cache_t* cache, const void* q, const int32_t* indices,
+                                        const int32_t* counts, int32_t n_cap, const resa_params_t* params,
+                                        void* out, float* lse, int32_t num_splits, void* stream);
+
+/*
  * Synchronises `stream`, then copies device_status[0..1] to *code_out /
  * *detail_out (either may be NULL) and clears device_status. Returns
  * RESA_ERR_DEVICE if a device error had been recorded, RESA_OK otherwise.

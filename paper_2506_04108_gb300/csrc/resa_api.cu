@@ -9,6 +9,7 @@
 #include <cmath>
 #include <cstdint>
 #include <cstring>
+#include <mutex>
 
 #include "resa.h"
 #include "resa_launch.h"
@@ -342,6 +343,67 @@ resa_status_t resa_rectify_attention(const resa_cache_t* cache, const void* q_ne
   cudaError_t e = launch_rectify(view(cache), tk, tv, static_cast<const uint16_t*>(q_new),
                                  static_cast<const uint16_t*>(k_new), static_cast<const uint16_t*>(v_new), f,
                                  scale_of(cache, params), splits, o_part, lse_part, st);
+  if (e == cudaSuccess)
+    e = launch_merge(o_part, lse_part, static_cast<int>(rows), splits, static_cast<uint16_t*>(out), lse, st);
+  return e == cudaSuccess ? RESA_OK : RESA_ERR_CUDA;
+}
+
+}  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Static scratch for resa_sparse_decode_static (callers that cannot allocate).
+// In host code `g_static_scratch` names a host-side stand-in, not the device
+// buffer, so its device address is looked up once per device with
+// cudaGetSymbolAddress (that device current) and passed to the kernels.
+// ---------------------------------------------------------------------------
+static __device__ __align__(256) unsigned char g_static_scratch[RESA_STATIC_SCRATCH_BYTES];
+
+namespace {
+std::mutex g_static_mu;
+void* g_static_ptr[resa::kMaxDevices];
+
+resa_status_t static_scratch_address(void** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return RESA_ERR_CUDA;
+  if (dev >= resa::kMaxDevices) return RESA_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  if (g_static_ptr[dev] == nullptr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || p == nullptr) return RESA_ERR_CUDA;
+    g_static_ptr[dev] = p;
+  }
+  *out = g_static_ptr[dev];
+  return RESA_OK;
+}
+}  // namespace
+
+extern "C" {
+
+resa_status_t resa_sparse_decode_static(const resa_cache_t* cache, const void* q, const int32_t* indices,
+                                        const int32_t* counts, int32_t n_cap, const resa_params_t* params,
+                                        void* out, float* lse, int32_t num_splits, void* stream) {
+  resa_status_t s = check_cache(cache);
+  if (s != RESA_OK) return s;
+  if ((s = check_params(params)) != RESA_OK) return s;
+  if (q == nullptr || indices == nullptr || counts == nullptr || out == nullptr || n_cap <= 0 || num_splits < 0)
+    return RESA_ERR_INVALID_ARG;
+  if (!aligned16(q)) return RESA_ERR_INVALID_ARG;
+  int splits = num_splits;
+  if (splits == 0 && (s = auto_decode_splits(cache, n_cap, &splits)) != RESA_OK) return s;
+  if (splits > 1024) return RESA_ERR_INVALID_ARG;
+  const size_t rows = static_cast<size_t>(cache->batch) * cache->num_q_heads;
+  if (partial_bytes(rows, splits) > RESA_STATIC_SCRATCH_BYTES) return RESA_ERR_WORKSPACE;
+  void* scratch = nullptr;
+  if ((s = static_scratch_address(&scratch)) != RESA_OK) return s;
+  CUtensorMap tk, tv;
+  if ((s = pool_tensor_map(cache, cache->k_pool, &tk)) != RESA_OK) return s;
+  if ((s = pool_tensor_map(cache, cache->v_pool, &tv)) != RESA_OK) return s;
+  float* o_part = static_cast<float*>(scratch);
+  float* lse_part = reinterpret_cast<float*>(static_cast<char*>(scratch) +
+                                             align_up(rows * splits * kHeadDimHost * sizeof(float)));
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  cudaError_t e = launch_sparse_decode(view(cache), tk, tv, static_cast<const uint16_t*>(q), indices, counts, n_cap,
+                                       scale_of(cache, params), splits, o_part, lse_part, st);
   if (e == cudaSuccess)
     e = launch_merge(o_part, lse_part, static_cast<int>(rows), splits, static_cast<uint16_t*>(out), lse, st);
   return e == cudaSuccess ? RESA_OK : RESA_ERR_CUDA;

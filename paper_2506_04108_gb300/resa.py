@@ -26,7 +26,7 @@ DEVICE_ERRORS = {0: "RESA_DEV_OK", 1: "RESA_DEV_SEQ_LEN_RANGE", 2: "RESA_DEV_PAG
                  3: "RESA_DEV_BUDGET_OVER_CAP", 4: "RESA_DEV_WAIT_TIMEOUT", 5: "RESA_DEV_BAD_INDEX"}
 EXPORTED = ["resa_abi_version", "resa_status_string", "resa_max_selected", "resa_decode_num_splits",
             "resa_workspace_size", "resa_update_summaries", "resa_commit_kv", "resa_select_blocks",
-            "resa_sparse_decode", "resa_rectify_attention", "resa_read_device_error"]
+            "resa_sparse_decode", "resa_rectify_attention", "resa_read_device_error", "resa_sparse_decode_static"]
 
 
 class ResaError(RuntimeError):
@@ -72,6 +72,7 @@ def load() -> ctypes.CDLL:
         "resa_sparse_decode": ([cp, pp, pp, pp, c_int32, pc, pp, pp, c_int32, pp, c_size_t, pp], c_int32),
         "resa_rectify_attention": ([cp, pp, pp, pp, c_int32, pc, pp, pp, pp, c_size_t, pp], c_int32),
         "resa_read_device_error": ([cp, POINTER(c_int32), POINTER(c_int32), pp], c_int32),
+        "resa_sparse_decode_static": ([cp, pp, pp, pp, c_int32, pc, pp, pp, c_int32, pp], c_int32),
     }
     for name, (args, ret) in sig.items():
         fn = getattr(L, name)
@@ -155,6 +156,16 @@ def resa_sparse_decode(cache: ResaCacheT, q, indices, counts, n_cap: int, p: Res
     _check(load().resa_sparse_decode(ctypes.byref(cache), _ptr(q), _ptr(indices), _ptr(counts), n_cap,
                                      ctypes.byref(p), _ptr(out), _ptr(lse), num_splits, _ptr(workspace),
                                      workspace_bytes, _stream(stream)), "resa_sparse_decode")
+
+
+def resa_sparse_decode_static(cache: ResaCacheT, q, indices, counts, n_cap: int, p: ResaParamsT, out, lse,
+                              num_splits: int, stream=None):
+    """resa_sparse_decode for callers that cannot allocate device memory: no
+    workspace argument; the split partials go to the library's static device
+    buffer (RESA_STATIC_SCRATCH_BYTES). Calls must not overlap on the GPU."""
+    _check(load().resa_sparse_decode_static(ctypes.byref(cache), _ptr(q), _ptr(indices), _ptr(counts), n_cap,
+                                            ctypes.byref(p), _ptr(out), _ptr(lse), num_splits, _stream(stream)),
+           "resa_sparse_decode_static")
 
 
 def resa_rectify_attention(cache: ResaCacheT, q_new, k_new, v_new, f: int, p: ResaParamsT, out, lse, workspace,
