@@ -48,6 +48,8 @@ __device__ __forceinline__ size_t summ_off(const CacheView& c, int b, int h, int
 
 __global__ void __launch_bounds__(256) commit_append_kernel(CacheView c, const uint16_t* __restrict__ k_new,
                                                             const uint16_t* __restrict__ v_new, int n) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int b = blockIdx.x;
   const int T = c.seq_lens[b];
   const int cap = c.max_blocks * kBlock;
@@ -101,6 +103,8 @@ __global__ void __launch_bounds__(256) commit_append_kernel(CacheView c, const u
 
 __global__ void __launch_bounds__(256) commit_overwrite_kernel(CacheView c, const uint16_t* __restrict__ k_new,
                                                                const uint16_t* __restrict__ v_new, int n) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int b = blockIdx.y;
   const int T = c.seq_lens[b];
   const int cap = c.max_blocks * kBlock;
@@ -149,6 +153,8 @@ __global__ void __launch_bounds__(256) commit_overwrite_kernel(CacheView c, cons
 // One warp per (sequence, head, block): lanes 0-15 take rows 0-7, lanes 16-31
 // rows 8-15, each lane one 16-byte chunk (8 dims); halves combine by shuffle.
 __global__ void __launch_bounds__(256) update_summaries_kernel(CacheView c, int begin, int end) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int b = blockIdx.z, h = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int blk = begin + blockIdx.x * 8 + warp;
@@ -196,13 +202,9 @@ __global__ void __launch_bounds__(256) update_summaries_kernel(CacheView c, int 
 cudaError_t launch_commit(const CacheView& c, const uint16_t* k_new, const uint16_t* v_new, int n, bool overwrite,
                           cudaStream_t st) {
   if (n == 0) return cudaSuccess;
-  if (!overwrite) {
-    commit_append_kernel<<<c.B, 256, 0, st>>>(c, k_new, v_new, n);
-  } else {
-    const dim3 grid((n + kBlock - 1) / kBlock + 1, c.B);
-    commit_overwrite_kernel<<<grid, 256, 0, st>>>(c, k_new, v_new, n);
-  }
-  return cudaGetLastError();
+  if (!overwrite) return launch_pdl(commit_append_kernel, dim3(c.B), dim3(256), 0, st, c, k_new, v_new, n);
+  const dim3 grid((n + kBlock - 1) / kBlock + 1, c.B);
+  return launch_pdl(commit_overwrite_kernel, grid, dim3(256), 0, st, c, k_new, v_new, n);
 }
 
 cudaError_t launch_update_summaries(const CacheView& c, int begin, int end, cudaStream_t st) {
@@ -210,8 +212,7 @@ cudaError_t launch_update_summaries(const CacheView& c, int begin, int end, cuda
   const int nblk = last - begin;
   if (nblk <= 0) return cudaSuccess;
   const dim3 grid((nblk + 7) / 8, c.Hkv, c.B);
-  update_summaries_kernel<<<grid, 256, 0, st>>>(c, begin, end);
-  return cudaGetLastError();
+  return launch_pdl(update_summaries_kernel, grid, dim3(256), 0, st, c, begin, end);
 }
 
 }  // namespace resa

@@ -52,6 +52,17 @@ __global__ void __launch_bounds__(kWarps * 32, 1) rectify_kernel(const __grid_co
   const int b = bh / c.Hkv, h = bh % c.Hkv;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int f = a.f, g = c.g;
+  const uint32_t sbase = smem_u32(smem);
+  const uint32_t bar0 = smem_u32(bars);
+  if (tid == 0) {
+    for (int st = 0; st < kStages; ++st) mbar_init(bar0 + 8 * st, 1);
+    fence_mbar_init();
+    prefetch_tmap(&tm_k);
+    prefetch_tmap(&tm_v);
+  }
+  __syncthreads();
+  pdl_launch_dependents();
+  pdl_wait();
   const int T = c.seq_lens[b];
   if (T < f || T > c.max_blocks * kBlock) {
     if (tid == 0 && s == 0 && rg == 0) record_error(c.status, RESA_DEV_SEQ_LEN_RANGE, b);
@@ -64,16 +75,6 @@ __global__ void __launch_bounds__(kWarps * 32, 1) rectify_kernel(const __grid_co
   const int n_pref = max(0, min(ntp, t0 + per) - t0);
   const int n_tail = (s == a.splits - 1) ? (f + kTile - 1) / kTile : 0;
   const int R = g * f;
-
-  const uint32_t sbase = smem_u32(smem);
-  const uint32_t bar0 = smem_u32(bars);
-  if (tid == 0) {
-    for (int st = 0; st < kStages; ++st) mbar_init(bar0 + 8 * st, 1);
-    fence_mbar_init();
-    prefetch_tmap(&tm_k);
-    prefetch_tmap(&tm_v);
-  }
-  __syncthreads();
 
   auto issue = [&](int lt, int st) {  // thread 0: prefix tile t0 + lt into stage st
     const int kb = (t0 + lt) * kTile;
@@ -312,8 +313,7 @@ cudaError_t launch_rectify(const CacheView& c, const CUtensorMap& tm_k, const CU
   if (e != cudaSuccess) return e;
   RectArgs a{q_new, k_new, v_new, f, splits, sm_scale * 1.44269504088896340736f, o_part, lse_part};
   const dim3 grid(splits, rectify_row_groups(c.g, f), c.B * c.Hkv);
-  rectify_kernel<<<grid, kWarps * 32, kSmem, st>>>(tm_k, tm_v, c, a);
-  return cudaGetLastError();
+  return launch_pdl(rectify_kernel, grid, dim3(kWarps * 32), kSmem, st, tm_k, tm_v, c, a);
 }
 
 }  // namespace resa

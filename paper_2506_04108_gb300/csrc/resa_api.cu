@@ -91,6 +91,7 @@ resa_status_t check_cache(const resa_cache_t* c) {
   // row coordinates of the pool and 32-bit index arithmetic must not overflow
   if (static_cast<int64_t>(c->num_pages) * c->num_kv_heads * c->block_size > INT32_MAX) return RESA_ERR_UNSUPPORTED;
   if (static_cast<int64_t>(c->max_blocks_per_seq) * c->block_size > INT32_MAX / 2) return RESA_ERR_UNSUPPORTED;
+  if (c->max_blocks_per_seq > select_max_blocks()) return RESA_ERR_UNSUPPORTED;
   if (c->k_pool == nullptr || c->v_pool == nullptr || c->page_table == nullptr || c->seq_lens == nullptr ||
       c->summaries == nullptr || c->device_status == nullptr)
     return RESA_ERR_INVALID_ARG;
@@ -139,10 +140,11 @@ resa_status_t auto_decode_splits(const resa_cache_t* c, int n_cap, int* out) {
   int sms = 0;
   const resa_status_t s = sm_count(&sms);
   if (s != RESA_OK) return s;
-  // Algorithm 2's num_splits: about two CTAs per SM over batch * KV heads,
-  // with at least two selected blocks per split.
+  // Algorithm 2's num_splits: as many splits as fit in one wave of resident
+  // decode CTAs over batch * KV heads (no tail wave), with at least two
+  // selected blocks per split.
   const int units = c->batch * c->num_kv_heads;
-  int splits = (2 * sms + units - 1) / units;
+  int splits = sms * decode_ctas_per_sm() / units;
   const int max_by_blocks = n_cap / 2 > 1 ? n_cap / 2 : 1;
   if (splits > max_by_blocks) splits = max_by_blocks;
   if (splits > 256) splits = 256;
@@ -285,9 +287,11 @@ resa_status_t resa_select_blocks(const resa_cache_t* cache, const void* q, const
   if (q == nullptr || indices == nullptr || counts == nullptr || n_cap <= 0) return RESA_ERR_INVALID_ARG;
   if (!aligned16(q)) return RESA_ERR_INVALID_ARG;
   if (workspace == nullptr || workspace_bytes < scores_bytes(cache)) return RESA_ERR_WORKSPACE;
+  int sms = 0;
+  if ((s = sm_count(&sms)) != RESA_OK) return s;
   const cudaError_t e = launch_select(view(cache), static_cast<const uint16_t*>(q), params->keep_ratio,
                                       params->n_min_blocks, params->n_local_blocks, indices, counts, n_cap,
-                                      static_cast<float*>(workspace), static_cast<cudaStream_t>(stream));
+                                      static_cast<float*>(workspace), sms, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? RESA_OK : RESA_ERR_CUDA;
 }
 

@@ -31,6 +31,16 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// --------------------------------------------- programmatic dependent launch ---
+// Every kernel is launched with programmatic stream serialization: it lets the
+// next kernel on the stream start launching (launch_dependents), and waits for
+// the previous kernel's completion and memory (wait) before touching any
+// global data, so only launch latency and shared-memory set-up overlap.
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // ------------------------------------------------------------ smem addr ---
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));

@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "resa.h"
 
 namespace resa {
@@ -25,6 +27,24 @@ struct CacheView {
   int32_t* status;
 };
 
+// Launches `kernel` with programmatic stream serialization (see
+// pdl_launch_dependents / pdl_wait in resa_device.cuh).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 // Sets cudaFuncAttributeMaxDynamicSharedMemorySize of `func` once per device
 // (kernel-launch paths then make no attribute calls, e.g. under graph capture).
 cudaError_t ensure_smem_attr(const void* func, int bytes, int slot);
@@ -36,10 +56,13 @@ cudaError_t launch_update_summaries(const CacheView& c, int block_begin, int blo
 
 // select.cu
 size_t select_smem_bytes(int max_blocks);
+int select_max_blocks();  // largest max_blocks_per_seq the selection supports
 cudaError_t launch_select(const CacheView& c, const uint16_t* q, double keep, int n_min, int n_local,
-                          int32_t* indices, int32_t* counts, int n_cap, float* scores, cudaStream_t st);
+                          int32_t* indices, int32_t* counts, int n_cap, float* scores, int sm_count,
+                          cudaStream_t st);
 
 // sparse_decode.cu
+int decode_ctas_per_sm();  // resident decode CTAs per SM (occupancy), >= 1
 cudaError_t launch_sparse_decode(const CacheView& c, const CUtensorMap& tm_k, const CUtensorMap& tm_v,
                                  const uint16_t* q, const int32_t* indices, const int32_t* counts, int n_cap,
                                  float sm_scale, int splits, float* o_part, float* lse_part, cudaStream_t st);

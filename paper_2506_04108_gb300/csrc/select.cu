@@ -6,14 +6,19 @@
 //               16-byte chunk (8 dims) of k_min and k_max, so a warp reads two
 //               contiguous 512-byte summaries per load instruction. The
 //               128-dim sum is a fixed-order butterfly over the 16 lanes.
-// topn_kernel   grid (KV head, sequence), 1024 threads. The n of Eq. 5 is
+// topn_kernel   one 8-CTA cluster per (sequence, KV head). The n of Eq. 5 is
 //               evaluated on the device from the device-resident length. The
 //               n-th largest order-preserving key is found by an 8-bit radix
-//               select (4 histogram passes over keys staged in shared
-//               memory, warp-aggregated atomics), then the selected ids are
-//               written in ascending order by a ballot compaction that also
-//               resolves ties at the threshold toward the lower block index.
-//               The last n_local blocks carry the maximum key (score +inf).
+//               select over keys staged in the CTAs' shared memory, with the
+//               histograms summed across the cluster through distributed
+//               shared memory; the selected ids are written in ascending order
+//               by a ballot compaction that resolves ties at the threshold
+//               toward the lower block index. The last n_local blocks carry
+//               the maximum key (score +inf).
+#include <cooperative_groups.h>
+
+#include <atomic>
+
 #include "resa_device.cuh"
 #include "resa_launch.h"
 
@@ -23,9 +28,10 @@ namespace {
 constexpr int kScoreWarps = 8;
 constexpr int kScoreUnroll = 4;                                    // 2 blocks per warp per step
 constexpr int kBlocksPerScoreCta = kScoreWarps * 2 * kScoreUnroll;  // 64
-constexpr int kTopnThreads = 1024;
+constexpr int kTopnCluster = 8;                                   // CTAs per (sequence, KV head)
+constexpr int kTopnThreads = 256;
 constexpr int kTopnWarps = kTopnThreads / 32;
-constexpr int kKeysInSmem = 32768;                                 // 128 KB of staged keys
+constexpr int kTopnSmemMax = 200 * 1024;                           // staged keys per CTA, bytes
 
 __device__ __forceinline__ float quest_term8(const float* q, const uint4& mn, const uint4& mx) {
   const uint32_t a[4] = {mn.x, mn.y, mn.z, mn.w};
@@ -39,16 +45,48 @@ __device__ __forceinline__ float quest_term8(const float* q, const uint4& mn, co
   return s;
 }
 
+// Loads of one CTA iteration: 8 warps x 2 half-warps x kScoreUnroll blocks.
+struct SummaryChunk {
+  uint4 mn[kScoreUnroll], mx[kScoreUnroll];
+};
+
+__device__ __forceinline__ void load_chunk(SummaryChunk& r, const uint16_t* sb, int base, int end, int warp,
+                                           int half, int ch) {
+#pragma unroll
+  for (int u = 0; u < kScoreUnroll; ++u) {
+    const int blk = base + warp * (2 * kScoreUnroll) + 2 * u + half;
+    if (blk < end) {
+      const uint16_t* s = sb + static_cast<size_t>(blk) * 2 * kHeadDim + ch * 8;
+      r.mn[u] = *reinterpret_cast<const uint4*>(s);
+      r.mx[u] = *reinterpret_cast<const uint4*>(s + kHeadDim);
+    } else {
+      r.mn[u] = make_uint4(0, 0, 0, 0);
+      r.mx[u] = make_uint4(0, 0, 0, 0);
+    }
+  }
+}
+
+// Grid (chunks, KV head, sequence) sized to one wave; CTA x scores the blocks
+// [x * per, min(M, (x + 1) * per)) of its (sequence, head), per = ceil(M /
+// chunks), 64 blocks per iteration. The next iteration's summaries are
+// loaded before the current one is reduced, and the first loads are issued
+// before the group's queries are read.
 __global__ void __launch_bounds__(256) score_kernel(CacheView c, const uint16_t* __restrict__ q,
-                                                    float* __restrict__ scores) {
+                                                    float* __restrict__ scores, int chunks) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int b = blockIdx.z, h = blockIdx.y;
   const int T = c.seq_lens[b];
   if (T < 0 || T > c.max_blocks * kBlock) return;  // reported by topn_kernel
   const int M = (T + kBlock - 1) / kBlock;
-  const int base = blockIdx.x * kBlocksPerScoreCta;
-  if (base >= M) return;
+  const int per = (M + chunks - 1) / chunks;
+  const int start = blockIdx.x * per, end = min(M, start + per);
+  if (start >= end) return;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int ch = lane & 15, half = lane >> 4;
+  const uint16_t* sb = c.summ + (static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks * 2 * kHeadDim;
+  SummaryChunk cur, nxt;
+  load_chunk(cur, sb, start, end, warp, half, ch);
 
   // pooled query (mean of the group's heads) for this lane's 8 dims
   float qp[8];
@@ -68,30 +106,21 @@ __global__ void __launch_bounds__(256) score_kernel(CacheView c, const uint16_t*
 #pragma unroll
   for (int j = 0; j < 8; ++j) qp[j] = qp[j] * inv_g;
 
-  const uint16_t* sb = c.summ + (static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks * 2 * kHeadDim;
-  uint4 mn[kScoreUnroll], mx[kScoreUnroll];
-  int blk[kScoreUnroll];
-#pragma unroll
-  for (int u = 0; u < kScoreUnroll; ++u) {
-    blk[u] = base + warp * (2 * kScoreUnroll) + 2 * u + half;
-    if (blk[u] < M) {
-      const uint16_t* s = sb + static_cast<size_t>(blk[u]) * 2 * kHeadDim + ch * 8;
-      mn[u] = *reinterpret_cast<const uint4*>(s);
-      mx[u] = *reinterpret_cast<const uint4*>(s + kHeadDim);
-    } else {
-      mn[u] = make_uint4(0, 0, 0, 0);
-      mx[u] = make_uint4(0, 0, 0, 0);
-    }
-  }
   float* out = scores + (static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks;
+  for (int base = start; base < end; base += kBlocksPerScoreCta) {
+    const bool more = base + kBlocksPerScoreCta < end;
+    if (more) load_chunk(nxt, sb, base + kBlocksPerScoreCta, end, warp, half, ch);
 #pragma unroll
-  for (int u = 0; u < kScoreUnroll; ++u) {
-    float s = quest_term8(qp, mn[u], mx[u]);
-    s += __shfl_xor_sync(0xffffffffu, s, 8);
-    s += __shfl_xor_sync(0xffffffffu, s, 4);
-    s += __shfl_xor_sync(0xffffffffu, s, 2);
-    s += __shfl_xor_sync(0xffffffffu, s, 1);
-    if (ch == 0 && blk[u] < M) out[blk[u]] = s;
+    for (int u = 0; u < kScoreUnroll; ++u) {
+      const int blk = base + warp * (2 * kScoreUnroll) + 2 * u + half;
+      float sc = quest_term8(qp, cur.mn[u], cur.mx[u]);
+      sc += __shfl_xor_sync(0xffffffffu, sc, 8);
+      sc += __shfl_xor_sync(0xffffffffu, sc, 4);
+      sc += __shfl_xor_sync(0xffffffffu, sc, 2);
+      sc += __shfl_xor_sync(0xffffffffu, sc, 1);
+      if (ch == 0 && blk < end) out[blk] = sc;
+    }
+    if (more) cur = nxt;
   }
 }
 
@@ -101,41 +130,56 @@ __device__ __forceinline__ uint32_t score_key(float s) {
   return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
-// Exclusive scan of one value per warp (kTopnWarps values) by warp 0.
-__device__ __forceinline__ void scan_warp_totals(int* vals, int* total) {
+// Exclusive scan of one int per warp (kTopnWarps values, in place) by warp 0.
+__device__ __forceinline__ void scan_warp_totals(int* vals) {
   const int lane = threadIdx.x & 31;
   if (threadIdx.x < 32) {
-    const int v = vals[lane];
+    const int v = lane < kTopnWarps ? vals[lane] : 0;
     int x = v;
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
+    for (int o = 1; o < kTopnWarps; o <<= 1) {
       const int y = __shfl_up_sync(0xffffffffu, x, o);
       if (lane >= o) x += y;
     }
-    vals[lane] = x - v;
-    if (lane == 31) *total = x;
+    if (lane < kTopnWarps) vals[lane] = x - v;
   }
 }
 
+// Cluster radix select, grid (kTopnCluster, KV head, sequence), one cluster
+// per (sequence, KV head). CTA r stages the order-preserving keys of blocks
+// [r * per, (r + 1) * per) in shared memory. Each 8-bit pass builds a local
+// histogram of the keys that still match the prefix; after one cluster
+// barrier every CTA sums the cluster's histograms through distributed shared
+// memory and finds the same digit (histograms are double-buffered by pass
+// parity, so one barrier per pass suffices). The select stops early when the
+// boundary bucket is taken whole. Then each CTA counts its keys above the
+// boundary and at it, reads the counts of the lower-ranked CTAs, and writes
+// its selected ids in ascending order (ties at the boundary to the lower id).
 __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const float* __restrict__ scores,
                                                             double keep, int n_min, int n_local,
                                                             int32_t* __restrict__ indices,
                                                             int32_t* __restrict__ counts, int n_cap) {
-  extern __shared__ uint32_t keys_smem[];
-  __shared__ int hist[256];
+  extern __shared__ uint32_t keys[];
+  __shared__ int hist[2][256];
+  __shared__ int tot[256];
   __shared__ int warp_a[kTopnWarps], warp_b[kTopnWarps];
-  __shared__ int sh_digit, sh_rem, sh_tot;
-
-  const int b = blockIdx.y, h = blockIdx.x;
+  __shared__ int sh_digit, sh_rem, sh_done, sh_eq_before, sh_sel_before;
+  __shared__ int cta_counts[2];  // keys above / at the boundary in this CTA, read by peers
+  namespace cg = cooperative_groups;
+  cg::cluster_group cluster = cg::this_cluster();
+  pdl_launch_dependents();
+  pdl_wait();
+  const int rank = static_cast<int>(cluster.block_rank());
+  const int b = blockIdx.z, h = blockIdx.y;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   int32_t* out = indices + (static_cast<size_t>(b) * c.Hkv + h) * n_cap;
   const int T = c.seq_lens[b];
-  if (T < 0 || T > c.max_blocks * kBlock) {
-    if (tid == 0) {
+  if (T < 0 || T > c.max_blocks * kBlock) {  // the whole cluster takes this branch
+    if (rank == 0 && tid == 0) {
       record_error(c.status, RESA_DEV_SEQ_LEN_RANGE, b);
       counts[b * c.Hkv + h] = 0;
     }
-    for (int i = tid; i < n_cap; i += kTopnThreads) out[i] = -1;
+    for (int i = rank * kTopnThreads + tid; i < n_cap; i += kTopnCluster * kTopnThreads) out[i] = -1;
     return;
   }
   const int M = (T + kBlock - 1) / kBlock;
@@ -146,48 +190,48 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
   nn = min(nn, static_cast<long long>(M));
   int n = static_cast<int>(nn);
   if (n > n_cap) {
-    if (tid == 0) record_error(c.status, RESA_DEV_BUDGET_OVER_CAP, b * c.Hkv + h);
+    if (rank == 0 && tid == 0) record_error(c.status, RESA_DEV_BUDGET_OVER_CAP, b * c.Hkv + h);
     n = n_cap;
   }
-  const float* sc = scores + (static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks;
-  const int first_forced = M - n_local;
-  const bool staged = c.max_blocks <= kKeysInSmem;  // the host sized the buffer from max_blocks
-  if (staged) {
-    for (int i = tid; i < M; i += kTopnThreads)
-      keys_smem[i] = (i >= first_forced) ? 0xFFFFFFFFu : score_key(sc[i]);
-  }
-  __syncthreads();
-  auto key_of = [&](int i) -> uint32_t {
-    if (staged) return keys_smem[i];
-    return (i >= first_forced) ? 0xFFFFFFFFu : score_key(sc[i]);
-  };
-  const int M_round = ((M + kTopnThreads - 1) / kTopnThreads) * kTopnThreads;
+  const int per = (M + kTopnCluster - 1) / kTopnCluster;
+  const int lo = rank * per, cnt = max(0, min(M, lo + per) - lo);
+  const float* sc = scores + (static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks + lo;
+  const int first_forced = M - n_local - lo;
+  for (int i = tid; i < cnt; i += kTopnThreads) keys[i] = (i >= first_forced) ? 0xFFFFFFFFu : score_key(sc[i]);
+  const int cnt_round = (cnt + 31) / 32 * 32;
 
-  // ---- radix select of the n-th largest key ----
+  // ---- radix select of the n-th largest key across the cluster ----
   uint32_t prefix = 0, pmask = 0;
   int rem = n;
+  __syncthreads();
   if (n > 0) {
     for (int pass = 0; pass < 4; ++pass) {
       const int shift = 24 - 8 * pass;
-      if (tid < 256) hist[tid] = 0;
+      int* hb = hist[pass & 1];
+      hb[tid] = 0;
       __syncthreads();
-      for (int i = tid; i < M_round; i += kTopnThreads) {
+      for (int i = tid; i < cnt_round; i += kTopnThreads) {
         uint32_t d = 0x100u;  // sentinel: not counted
-        if (i < M) {
-          const uint32_t k = key_of(i);
+        if (i < cnt) {
+          const uint32_t k = keys[i];
           if ((k & pmask) == prefix) d = (k >> shift) & 0xFFu;
         }
         const unsigned peers = __match_any_sync(0xffffffffu, d);
-        if (d != 0x100u && lane == __ffs(peers) - 1) atomicAdd(&hist[d], __popc(peers));
+        if (d != 0x100u && lane == __ffs(peers) - 1) atomicAdd(&hb[d], __popc(peers));
       }
+      cluster.sync();  // every CTA's histogram of this pass is complete and visible
+      int t = 0;
+#pragma unroll
+      for (int r = 0; r < kTopnCluster; ++r) t += cluster.map_shared_rank(hb, r)[tid];
+      tot[tid] = t;
       __syncthreads();
       if (warp == 0) {
         // lane l owns digits 255-8l ... 248-8l (descending)
-        int cnt[8], sum = 0;
+        int cn[8], sum = 0;
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
-          cnt[j] = hist[255 - 8 * lane - j];
-          sum += cnt[j];
+          cn[j] = tot[255 - 8 * lane - j];
+          sum += cn[j];
         }
         int incl = sum;
 #pragma unroll
@@ -200,12 +244,13 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
           int cum = excl;
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
-            if (cum + cnt[j] >= rem) {
+            if (cum + cn[j] >= rem) {
               sh_digit = 255 - 8 * lane - j;
               sh_rem = rem - cum;
+              sh_done = (rem - cum == cn[j]) ? 1 : 0;  // the whole bucket is taken
               break;
             }
-            cum += cnt[j];
+            cum += cn[j];
           }
         }
       }
@@ -213,23 +258,24 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
       prefix |= static_cast<uint32_t>(sh_digit) << shift;
       pmask |= 0xFFu << shift;
       rem = sh_rem;
+      if (sh_done) break;  // identical decision in every CTA of the cluster
     }
   }
-  // keys > prefix are all taken; of the keys == prefix, the `rem` lowest ids.
-  const uint32_t tau = prefix;
-  const int take_eq = (n > 0) ? rem : 0;
+  // Selected: (key & pmask) > prefix, or == prefix among the first `take_eq`
+  // such keys in block order.
+  const int take_eq = n > 0 ? rem : 0;
 
-  // ---- ordered compaction: each warp owns a contiguous id range ----
-  const int per_warp = ((M + kTopnWarps * 32 - 1) / (kTopnWarps * 32)) * 32;
-  const int w0 = warp * per_warp, w1 = min(M, w0 + per_warp);
+  // ---- ordered compaction: warps own contiguous id ranges of the CTA ----
+  const int per_warp = (cnt_round / 32 + kTopnWarps - 1) / kTopnWarps * 32;
+  const int w0 = warp * per_warp, w1 = min(cnt, w0 + per_warp);
   int gt = 0, eq = 0;
   if (n > 0) {
     for (int i0 = w0; i0 < w0 + per_warp; i0 += 32) {
       const int i = i0 + lane;
-      const uint32_t k = (i < w1) ? key_of(i) : 0u;
       const bool in = i < w1;
-      gt += __popc(__ballot_sync(0xffffffffu, in && k > tau));
-      eq += __popc(__ballot_sync(0xffffffffu, in && k == tau));
+      const uint32_t k = in ? (keys[i] & pmask) : 0u;
+      gt += __popc(__ballot_sync(0xffffffffu, in && k > prefix));
+      eq += __popc(__ballot_sync(0xffffffffu, in && k == prefix));
     }
   }
   if (lane == 0) {
@@ -237,59 +283,108 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
     warp_b[warp] = gt;
   }
   __syncthreads();
-  scan_warp_totals(warp_a, &sh_tot);  // exclusive prefix of equal keys per warp
-  __syncthreads();
-  if (lane == 0) {
-    const int eq_before = warp_a[warp];
-    const int eq_taken = max(0, min(eq, take_eq - eq_before));
-    warp_b[warp] = gt + eq_taken;
+  if (tid == 0) {
+    int g2 = 0, e2 = 0;
+    for (int w = 0; w < kTopnWarps; ++w) {
+      g2 += warp_b[w];
+      e2 += warp_a[w];
+    }
+    cta_counts[0] = g2;
+    cta_counts[1] = e2;
+  }
+  cluster.sync();  // every CTA's counts are visible
+  if (tid == 0) {
+    int eq_before = 0, sel_before = 0;
+    for (int r = 0; r < rank; ++r) {
+      const int* pc = cluster.map_shared_rank(cta_counts, r);
+      const int g2 = pc[0], e2 = pc[1];
+      sel_before += g2 + max(0, min(e2, take_eq - eq_before));
+      eq_before += e2;
+    }
+    sh_eq_before = eq_before;
+    sh_sel_before = sel_before;
   }
   __syncthreads();
-  scan_warp_totals(warp_b, &sh_tot);  // exclusive prefix of selected ids per warp
+  scan_warp_totals(warp_a);  // exclusive prefix of equal keys per warp
+  __syncthreads();
+  if (lane == 0) {
+    const int eq_b = sh_eq_before + warp_a[warp];
+    warp_b[warp] = gt + max(0, min(eq, take_eq - eq_b));
+  }
+  __syncthreads();
+  scan_warp_totals(warp_b);  // exclusive prefix of selected ids per warp
   __syncthreads();
   if (n > 0) {
-    int eq_seen = warp_a[warp];
-    int pos = warp_b[warp];
+    int eq_seen = sh_eq_before + warp_a[warp];
+    int pos = sh_sel_before + warp_b[warp];
     for (int i0 = w0; i0 < w0 + per_warp; i0 += 32) {
       const int i = i0 + lane;
       const bool in = i < w1;
-      const uint32_t k = in ? key_of(i) : 0u;
-      const bool is_eq = in && k == tau;
+      const uint32_t k = in ? (keys[i] & pmask) : 0u;
+      const bool is_eq = in && k == prefix;
       const unsigned eqm = __ballot_sync(0xffffffffu, is_eq);
       const int my_eq_rank = eq_seen + __popc(eqm & ((1u << lane) - 1u));
-      const bool sel = in && (k > tau || (is_eq && my_eq_rank < take_eq));
+      const bool sel = in && (k > prefix || (is_eq && my_eq_rank < take_eq));
       const unsigned selm = __ballot_sync(0xffffffffu, sel);
-      if (sel) out[pos + __popc(selm & ((1u << lane) - 1u))] = i;
+      if (sel) out[pos + __popc(selm & ((1u << lane) - 1u))] = lo + i;
       eq_seen += __popc(eqm);
       pos += __popc(selm);
     }
   }
-  for (int i = n + tid; i < n_cap; i += kTopnThreads) out[i] = -1;
-  if (tid == 0) counts[b * c.Hkv + h] = n;
+  for (int i = n + rank * kTopnThreads + tid; i < n_cap; i += kTopnCluster * kTopnThreads) out[i] = -1;
+  if (rank == 0 && tid == 0) counts[b * c.Hkv + h] = n;
+  cluster.sync();  // no CTA leaves while a peer may still read its counts
 }
 
 }  // namespace
 
 size_t select_smem_bytes(int max_blocks) {
-  const int staged = max_blocks <= kKeysInSmem ? max_blocks : 0;
-  return static_cast<size_t>(staged) * sizeof(uint32_t);
+  return static_cast<size_t>((max_blocks + kTopnCluster - 1) / kTopnCluster) * sizeof(uint32_t);
 }
 
+int select_max_blocks() { return kTopnCluster * (kTopnSmemMax / static_cast<int>(sizeof(uint32_t))); }
+
 cudaError_t launch_select(const CacheView& c, const uint16_t* q, double keep, int n_min, int n_local,
-                          int32_t* indices, int32_t* counts, int n_cap, float* scores, cudaStream_t st) {
-  const dim3 sgrid((c.max_blocks + kBlocksPerScoreCta - 1) / kBlocksPerScoreCta, c.Hkv, c.B);
-  score_kernel<<<sgrid, kScoreWarps * 32, 0, st>>>(c, q, scores);
-  cudaError_t e = cudaGetLastError();
+                          int32_t* indices, int32_t* counts, int n_cap, float* scores, int sm_count,
+                          cudaStream_t st) {
+  // one wave of resident score CTAs, shared by batch * KV heads
+  static std::atomic<int> occ_cache{0};
+  int occ = occ_cache.load(std::memory_order_relaxed);
+  if (occ == 0) {
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, score_kernel, kScoreWarps * 32, 0) != cudaSuccess ||
+        occ < 1)
+      occ = 1;
+    occ_cache.store(occ, std::memory_order_relaxed);
+  }
+  const int units = c.B * c.Hkv;
+  const int max_chunks = (c.max_blocks + kBlocksPerScoreCta - 1) / kBlocksPerScoreCta;
+  int chunks = occ * sm_count / units;
+  if (chunks > max_chunks) chunks = max_chunks;
+  if (chunks < 1) chunks = 1;
+  cudaError_t e = launch_pdl(score_kernel, dim3(chunks, c.Hkv, c.B), dim3(kScoreWarps * 32), 0, st, c, q, scores,
+                             chunks);
   if (e != cudaSuccess) return e;
   const size_t smem = select_smem_bytes(c.max_blocks);
   if (smem > 48 * 1024) {
-    // sized for the largest staging buffer so one attribute call serves every cache
-    e = ensure_smem_attr(reinterpret_cast<const void*>(topn_kernel), select_smem_bytes(kKeysInSmem), 2);
+    e = ensure_smem_attr(reinterpret_cast<const void*>(topn_kernel), kTopnSmemMax, 2);
     if (e != cudaSuccess) return e;
   }
-  topn_kernel<<<dim3(c.Hkv, c.B), kTopnThreads, smem, st>>>(c, scores, keep, n_min, n_local, indices, counts,
-                                                            n_cap);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(kTopnCluster, c.Hkv, c.B);
+  cfg.blockDim = dim3(kTopnThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = kTopnCluster;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, topn_kernel, c, static_cast<const float*>(scores), keep, n_min, n_local, indices,
+                            counts, n_cap);
 }
 
 }  // namespace resa

@@ -18,6 +18,8 @@
 //   * The 4 warps' (m, l, O) are merged through shared memory; the CTA writes
 //     a normalised partial O (fp32) and its log2-sum-exp for each head.
 // merge_kernel, one CTA per output row: LSE-weighted sum of the split partials.
+#include <atomic>
+
 #include "resa_device.cuh"
 #include "resa_launch.h"
 
@@ -54,6 +56,17 @@ __global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid
 
   const int s = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t ring = smem_u32(smem) + warp * kStages * kStageBytes;
+  const uint32_t bar0 = smem_u32(bars + warp * kStages);
+  if (lane == 0) {
+    for (int st = 0; st < kStages; ++st) mbar_init(bar0 + 8 * st, 1);
+    fence_mbar_init();
+    prefetch_tmap(&tm_k);
+    prefetch_tmap(&tm_v);
+  }
+  __syncwarp();
+  pdl_launch_dependents();
+  pdl_wait();
   const int T = c.seq_lens[b];
   int n = a.counts[b * c.Hkv + h];
   if (T < 0 || T > c.max_blocks * kBlock) {
@@ -70,25 +83,28 @@ __global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid
   const int cnt = nj > warp ? (nj - warp + kWarps - 1) / kWarps : 0;
   const int32_t* idx = a.indices + static_cast<size_t>(b * c.Hkv + h) * a.n_cap + j0 + warp;
 
-  const uint32_t ring = smem_u32(smem) + warp * kStages * kStageBytes;
-  const uint32_t bar0 = smem_u32(bars + warp * kStages);
-  if (lane == 0) {
-    for (int st = 0; st < kStages; ++st) mbar_init(bar0 + 8 * st, 1);
-    fence_mbar_init();
-  }
-  __syncwarp();
-
-  // Page of the it-th block of this warp, or -1 if the block id or its page
-  // is out of range (the block is then treated as fully masked).
-  auto page_of = [&](int it, int& blk) -> int {
+  // Block id and page of the warp's it-th block; the first 32 are resolved by
+  // all lanes at once (two round trips), later ones on demand. page = -1: the
+  // block id is out of range; -2: its page is. Such blocks are fully masked.
+  auto resolve = [&](int it, int& blk) -> int {
     blk = idx[it * kWarps];
     if (blk < 0 || blk >= M) return -1;
     const int page = c.page_table[static_cast<size_t>(b) * c.max_blocks + blk];
     return (page >= 0 && page < c.num_pages) ? page : -2;
   };
-  auto issue = [&](int it, int st) {  // lane 0 only
+  int pre_blk = -1, pre_page = -1;
+  if (lane < cnt) pre_page = resolve(lane, pre_blk);
+  auto info = [&](int it, int& blk) -> int {  // warp-uniform
+    if (it < 32) {
+      blk = __shfl_sync(0xffffffffu, pre_blk, it);
+      return __shfl_sync(0xffffffffu, pre_page, it);
+    }
+    return resolve(it, blk);
+  };
+  auto issue = [&](int it, int st) {  // warp-uniform; lane 0 issues
     int blk;
-    const int page = page_of(it, blk);
+    const int page = info(it, blk);
+    if (lane != 0) return;
     const uint32_t bar = bar0 + 8 * st;
     if (page < 0) {
       record_error(c.status, page == -1 ? RESA_DEV_BAD_INDEX : RESA_DEV_PAGE_RANGE, b * c.Hkv + h);
@@ -119,12 +135,7 @@ __global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid
   }
 
   int issued = 0;
-  if (lane == 0) {
-    prefetch_tmap(&tm_k);
-    prefetch_tmap(&tm_v);
-    for (; issued < min(kStages, cnt); ++issued) issue(issued, issued);
-  }
-  issued = __shfl_sync(0xffffffffu, issued, 0);
+  for (; issued < min(kStages, cnt); ++issued) issue(issued, issued);
 
   float m0 = kNegInf, m1 = kNegInf, l0 = 0.f, l1 = 0.f;
   float acc[8][4];
@@ -145,7 +156,7 @@ __global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid
     }
     mbar_try_wait(bar, par);  // acquire for every lane (the phase has completed)
     int blk;
-    const int page = page_of(it, blk);
+    const int page = info(it, blk);
     const int valid = page < 0 ? 0 : min(kBlock, T - blk * kBlock);
     const uint32_t kb = ring + st * kStageBytes, vb = kb + 4096;
     if (valid < kBlock) {  // rows past the end (or an invalid block) may hold garbage: zero V
@@ -210,10 +221,8 @@ __global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid
     }
     __syncwarp();
     if (issued < cnt) {
-      if (lane == 0) {
-        fence_proxy_async_smem();
-        issue(issued, st);
-      }
+      if (lane == 0) fence_proxy_async_smem();
+      issue(issued, st);
       ++issued;
     }
   }
@@ -277,44 +286,86 @@ __global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid
   }
 }
 
-__global__ void __launch_bounds__(128) merge_kernel(const float* __restrict__ o_part,
-                                                    const float* __restrict__ lse_part, int splits,
-                                                    uint16_t* __restrict__ out, float* __restrict__ lse_out) {
-  extern __shared__ float w[];
-  __shared__ float sh_m, sh_l;
+// One CTA of 8 warps per output row: every warp reduces the split
+// log2-sum-exps itself (shuffles, no barrier), then warp w accumulates the
+// splits w, w + 8, ... for 4 of the 128 dims per lane, four splits' loads in
+// flight at a time; the 8 partial rows are summed through shared memory.
+constexpr int kMergeWarps = 8;
+
+__global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const float* __restrict__ o_part,
+                                                                 const float* __restrict__ lse_part, int splits,
+                                                                 uint16_t* __restrict__ out,
+                                                                 float* __restrict__ lse_out) {
+  __shared__ float4 red[kMergeWarps][kHeadDim / 4];
+  pdl_launch_dependents();
+  pdl_wait();
   const size_t row = blockIdx.x;
-  const int t = threadIdx.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const float* lp = lse_part + row * splits;
-  if (t < 32) {
-    float m = kNegInf;
-    for (int s = t; s < splits; s += 32) m = fmaxf(m, lp[s]);
+  float m = kNegInf;
+  for (int s = lane; s < splits; s += 32) m = fmaxf(m, lp[s]);
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-    if (t == 0) sh_m = m;
-  }
-  __syncthreads();
-  const float M = sh_m;
-  for (int s = t; s < splits; s += 128) w[s] = (lp[s] == kNegInf) ? 0.f : exp2f(lp[s] - M);
-  __syncthreads();
-  if (t < 32) {
-    float l = 0.f;
-    for (int s = t; s < splits; s += 32) l += w[s];
+  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+  const float base = safe_base(m);
+  float l = 0.f;
+  for (int s = lane; s < splits; s += 32) l += exp2f(lp[s] - base);
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-    if (t == 0) sh_l = l;
+  for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+  const float4* op = reinterpret_cast<const float4*>(o_part + row * splits * kHeadDim) + lane;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int s0 = warp; s0 < splits; s0 += 4 * kMergeWarps) {
+    float4 v[4];
+    float w[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int s = s0 + u * kMergeWarps;
+      const bool ok = s < splits;
+      v[u] = ok ? op[s * (kHeadDim / 4)] : make_float4(0.f, 0.f, 0.f, 0.f);
+      w[u] = ok ? exp2f(lp[s] - base) : 0.f;
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      acc.x += w[u] * v[u].x;
+      acc.y += w[u] * v[u].y;
+      acc.z += w[u] * v[u].z;
+      acc.w += w[u] * v[u].w;
+    }
   }
+  red[warp][lane] = acc;
   __syncthreads();
-  const float L = sh_l;
-  const float inv = L > 0.f ? 1.f / L : 0.f;
-  const float* op = o_part + row * splits * kHeadDim + t;
-  float v = 0.f;
-  for (int s = 0; s < splits; ++s) v += w[s] * op[static_cast<size_t>(s) * kHeadDim];
-  const __nv_bfloat16 r = __float2bfloat16_rn(v * inv);
-  out[row * kHeadDim + t] = *reinterpret_cast<const uint16_t*>(&r);
-  if (lse_out != nullptr && t == 0) lse_out[row] = L > 0.f ? (M + log2f(L)) * 0.69314718055994530942f : kNegInf;
+  if (warp == 0) {
+    float4 t = red[0][lane];
+#pragma unroll
+    for (int w = 1; w < kMergeWarps; ++w) {
+      t.x += red[w][lane].x;
+      t.y += red[w][lane].y;
+      t.z += red[w][lane].z;
+      t.w += red[w][lane].w;
+    }
+    const float inv = l > 0.f ? 1.f / l : 0.f;
+    uint2 packed;
+    packed.x = pack_bf16x2(t.x * inv, t.y * inv);
+    packed.y = pack_bf16x2(t.z * inv, t.w * inv);
+    *reinterpret_cast<uint2*>(out + row * kHeadDim + 4 * lane) = packed;
+    if (lse_out != nullptr && lane == 0) lse_out[row] = l > 0.f ? (m + log2f(l)) * 0.69314718055994530942f : kNegInf;
+  }
 }
 
 }  // namespace
+
+int decode_ctas_per_sm() {
+  static std::atomic<int> cached{0};
+  int v = cached.load(std::memory_order_relaxed);
+  if (v > 0) return v;
+  if (ensure_smem_attr(reinterpret_cast<const void*>(sparse_decode_kernel), kDecodeSmem, 0) != cudaSuccess) return 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, sparse_decode_kernel, kWarps * 32, kDecodeSmem) !=
+          cudaSuccess ||
+      n < 1)
+    n = 1;
+  cached.store(n, std::memory_order_relaxed);
+  return n;
+}
 
 cudaError_t launch_sparse_decode(const CacheView& c, const CUtensorMap& tm_k, const CUtensorMap& tm_v,
                                  const uint16_t* q, const int32_t* indices, const int32_t* counts, int n_cap,
@@ -322,15 +373,15 @@ cudaError_t launch_sparse_decode(const CacheView& c, const CUtensorMap& tm_k, co
   cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(sparse_decode_kernel), kDecodeSmem, 0);
   if (e != cudaSuccess) return e;
   DecodeArgs a{q, indices, counts, n_cap, splits, sm_scale * 1.44269504088896340736f, o_part, lse_part};
-  sparse_decode_kernel<<<dim3(splits, c.Hkv, c.B), kWarps * 32, kDecodeSmem, st>>>(tm_k, tm_v, c, a);
-  return cudaGetLastError();
+  return launch_pdl(sparse_decode_kernel, dim3(splits, c.Hkv, c.B), dim3(kWarps * 32), kDecodeSmem, st, tm_k,
+                    tm_v, c, a);
 }
 
 cudaError_t launch_merge(const float* o_part, const float* lse_part, int rows, int splits, uint16_t* out,
                          float* lse_out, cudaStream_t st) {
   if (rows == 0) return cudaSuccess;
-  merge_kernel<<<rows, 128, splits * sizeof(float), st>>>(o_part, lse_part, splits, out, lse_out);
-  return cudaGetLastError();
+  return launch_pdl(merge_kernel, dim3(rows), dim3(kMergeWarps * 32), 0, st, o_part, lse_part, splits, out,
+                    lse_out);
 }
 
 }  // namespace resa
