@@ -1,31 +1,65 @@
-// Dense rectification attention (Section 2.2; Algorithm 1 DenseForward).
+// Dense rectification attention (Section 2.2; Algorithm 1 DenseForward) on
+// the 5th-generation tensor cores (tcgen05, accumulators in tensor memory).
 //
-// For each (sequence b, KV head h) the g*f query rows of the group (row
-// r = i*g + j: token i of the f, query head h*g + j, position T - f + i)
-// attend causally to the whole cache. Work split:
-//   grid (key splits, row groups of 128, sequence * KV head), 8 warps,
-//   warp w owns 16 query rows; the CTA streams 64-key tiles of the prefix
-//   [0, T - f) from the paged cache with bulk-tensor TMA (SWIZZLE_128B,
-//   one copy per 16-key page per 64-column half) into a 2-stage ring, and
-//   the last split also takes the f-token tail from k_new / v_new with the
-//   causal mask (key t of the tail is visible to token i iff t <= i).
-//   S = Q K^T and O += P V run on m16n8k16 bf16 MMAs with fp32 accumulation
-//   and an online softmax in the log2 domain; each split writes a
-//   normalised partial O and its log2-sum-exp, combined by merge_kernel.
+// Work: for each (sequence b, KV head h) the f most recent tokens' queries of
+// the group attend causally to the cache: query row i (position T - f + i)
+// sees positions [0, T - f + i]. Keys/values of the prefix [0, T - f) come
+// from the paged cache, those of the f tokens from k_new / v_new.
+//
+// Rows: r = 8 * i + j (token i, query head h*g + j; heads padded to 8, so for
+// g = 7 the M-tile count f/16 is the same as unpadded). A CTA owns up to two
+// 128-row M-tiles (256 rows) of one (b, h) and a contiguous range of 64-key
+// tiles (a key split); the last split also takes the causal tail. Partials
+// (normalised O, log2-sum-exp) are combined by merge_kernel.
+//
+// CTA = 12 warps:
+//   warp 0      TMA producer: 64-key K and V tiles of the prefix, one
+//               SWIZZLE_128B box per 16-key page per 64-column half, into a
+//               2-stage ring (kv_full / kv_empty mbarriers); the causal tail
+//               is written by the warp's lanes in the same swizzled layout.
+//   warp 1      allocates 512 TMEM columns; lane 0 issues the MMAs:
+//               S[t] = Q K^T (M 128, N 64, K 128; both operands K-major) into
+//               a double-buffered TMEM S, and O += P V (M 128, N 128, K 64;
+//               P K-major from shared memory, V MN-major) into TMEM O.
+//   warps 4-11  softmax: one thread per query row (TMEM lane), so the row max
+//               and sum need no shuffles. P is written to shared memory as
+//               bf16. O is rescaled in TMEM only when a row maximum grows by
+//               more than 2^8 (exact: the exponent base is carried along).
+// TMEM columns: O[mt] = [128 mt, 128 mt + 128), S[buf][mt] = 256 + 64 (2 buf + mt).
+// Every mbarrier wait is bounded; a wait that runs out records
+// RESA_DEV_WAIT_TIMEOUT and the CTA winds down, freeing its TMEM.
 #include "resa_device.cuh"
 #include "resa_launch.h"
 
 namespace resa {
 namespace {
 
-constexpr int kWarps = 8;
-constexpr int kRows = 16 * kWarps;  // query rows per CTA
-constexpr int kTile = 64;           // keys per tile
-constexpr int kHalfBytes = kTile * 128;       // one 64-column half of a tile
-constexpr int kStageBytes = 4 * kHalfBytes;   // K (2 halves) + V (2 halves) = 32 KB
+constexpr int kThreads = 384;
+constexpr int kSoftmaxWarp0 = 4;
+constexpr int kMTile = 128;
+constexpr int kMaxMTiles = 2;
+constexpr int kRowsPerCta = kMTile * kMaxMTiles;  // 256
+constexpr int kTileKeys = 64;
 constexpr int kStages = 2;
-constexpr int kSmem = kStages * kStageBytes + 1024 + 64;
+constexpr int kQHalf = kRowsPerCta * 128;          // [256 rows][64 dims] bf16 = 32 KB
+constexpr int kKVHalf = kTileKeys * 128;           // [64 keys][64 dims] = 8 KB
+constexpr int kStageBytes = 4 * kKVHalf;           // K (2 halves) + V (2 halves) = 32 KB
+constexpr int kPTile = kMTile * 128;               // [128 rows][64 keys] = 16 KB
+constexpr int kOffQ = 0;
+constexpr int kOffP = 2 * kQHalf;                  // 64 KB
+constexpr int kOffKV = kOffP + 2 * kMaxMTiles * kPTile;   // 128 KB
+constexpr int kOffBar = kOffKV + kStages * kStageBytes;  // 192 KB
+constexpr int kSmem = kOffBar + 256 + 1024;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kColO = 0;
+constexpr uint32_t kColS = 256;
+constexpr uint32_t kIdescS = idesc_bf16_f32(kMTile, kTileKeys, 0, 0);
+constexpr uint32_t kIdescO = idesc_bf16_f32(kMTile, 128, 0, 1);
+constexpr float kRescaleLog2 = 8.f;
 constexpr float kNegInf = -__builtin_huge_valf();
+
+// barrier slots (uint64) in the barrier region
+constexpr int kBarKvFull = 0, kBarKvEmpty = 2, kBarSFull = 4, kBarPFull = 6, kBarODone = 8, kBarFinal = 10;
 
 struct RectArgs {
   const uint16_t* q_new;  // [B][f][Hq][128]
@@ -40,271 +74,319 @@ struct RectArgs {
 
 __device__ __forceinline__ float safe_base(float m) { return m == kNegInf ? 0.f : m; }
 
-__global__ void __launch_bounds__(kWarps * 32, 1) rectify_kernel(const __grid_constant__ CUtensorMap tm_k,
-                                                                 const __grid_constant__ CUtensorMap tm_v,
-                                                                 CacheView c, RectArgs a) {
+// Warp-uniform bounded wait: lane 0 polls, the verdict is broadcast, and every
+// lane then observes the completed phase itself.
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity) {
+  int ok = 1;
+  if ((threadIdx.x & 31) == 0) ok = mbar_wait_bounded(bar, parity) ? 1 : 0;
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  if (ok) mbar_try_wait(bar, parity);
+  return ok != 0;
+}
+
+__global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_constant__ CUtensorMap tm_k,
+                                                              const __grid_constant__ CUtensorMap tm_v,
+                                                              CacheView c, RectArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
-  __shared__ int sh_ok;
+  const uint32_t sbase = smem_u32(smem);
+  const uint32_t bar0 = sbase + kOffBar;
+  auto bar = [&](int slot) -> uint32_t { return bar0 + 8u * slot; };
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kOffBar + 128);
 
   const int s = blockIdx.x, rg = blockIdx.y, bh = blockIdx.z;
   const int b = bh / c.Hkv, h = bh % c.Hkv;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int f = a.f, g = c.g;
-  const uint32_t sbase = smem_u32(smem);
-  const uint32_t bar0 = smem_u32(bars);
+  const int rows_total = 8 * f;
+  const int row0 = rg * kRowsPerCta;
+  const int MT = min(kMaxMTiles, (rows_total - row0 + kMTile - 1) / kMTile);
+
   if (tid == 0) {
-    for (int st = 0; st < kStages; ++st) mbar_init(bar0 + 8 * st, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(bar(kBarKvFull + i), 1);
+      mbar_init(bar(kBarKvEmpty + i), 1);
+      mbar_init(bar(kBarSFull + i), 1);
+      mbar_init(bar(kBarPFull + i), kMTile * MT);
+      mbar_init(bar(kBarODone + i), 1);
+    }
+    mbar_init(bar(kBarFinal), 1);
     fence_mbar_init();
     prefetch_tmap(&tm_k);
     prefetch_tmap(&tm_v);
   }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
   __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
   pdl_launch_dependents();
   pdl_wait();
+
   const int T = c.seq_lens[b];
-  if (T < f || T > c.max_blocks * kBlock) {
-    if (tid == 0 && s == 0 && rg == 0) record_error(c.status, RESA_DEV_SEQ_LEN_RANGE, b);
-    return;
-  }
-  const int P = T - f;                         // prefix keys from the cache
-  const int ntp = (P + kTile - 1) / kTile;     // prefix tiles
+  const bool bad = (T < f || T > c.max_blocks * kBlock);
+  const int P = T - f;  // prefix keys from the cache
+  const int ntp = bad ? 0 : (P + kTileKeys - 1) / kTileKeys;
   const int per = (ntp + a.splits - 1) / a.splits;
   const int t0 = s * per;
   const int n_pref = max(0, min(ntp, t0 + per) - t0);
-  const int n_tail = (s == a.splits - 1) ? (f + kTile - 1) / kTile : 0;
-  const int R = g * f;
+  const int n_tail = (!bad && s == a.splits - 1) ? (f + kTileKeys - 1) / kTileKeys : 0;
+  const int n_tiles = n_pref + n_tail;
+  if (bad && tid == 0 && s == 0 && rg == 0) record_error(c.status, RESA_DEV_SEQ_LEN_RANGE, b);
 
-  auto issue = [&](int lt, int st) {  // thread 0: prefix tile t0 + lt into stage st
-    const int kb = (t0 + lt) * kTile;
-    const uint32_t bar = bar0 + 8 * st;
-    const uint32_t dk = sbase + st * kStageBytes, dv = dk + 2 * kHalfBytes;
-    int pages = 0, rows[4];
-    for (int pg = 0; pg < 4; ++pg) {
-      rows[pg] = -1;
-      const int blk = kb / kBlock + pg;
-      if (blk * kBlock >= P) continue;
-      const int page = c.page_table[static_cast<size_t>(b) * c.max_blocks + blk];
-      if (page < 0 || page >= c.num_pages) {
-        record_error(c.status, RESA_DEV_PAGE_RANGE, b);
-        continue;
-      }
-      rows[pg] = (page * c.Hkv + h) * kBlock;
-      ++pages;
-    }
-    mbar_arrive_expect_tx(bar, pages * 4 * 2048);
-    for (int pg = 0; pg < 4; ++pg) {
-      if (rows[pg] < 0) continue;
-      const uint32_t o = pg * 2048;
-      tma_load_2d(dk + o, &tm_k, bar, 0, rows[pg]);
-      tma_load_2d(dk + kHalfBytes + o, &tm_k, bar, 64, rows[pg]);
-      tma_load_2d(dv + o, &tm_v, bar, 0, rows[pg]);
-      tma_load_2d(dv + kHalfBytes + o, &tm_v, bar, 64, rows[pg]);
-    }
-  };
-  if (tid == 0)
-    for (int lt = 0; lt < min(kStages, n_pref); ++lt) issue(lt, lt);
-
-  // Q rows of this thread: rA = row0 + 16*warp + lane/4, rB = rA + 8.
-  const int rA = rg * kRows + warp * 16 + (lane >> 2), rB = rA + 8;
-  const int iA = rA < R ? rA / g : -1, iB = rB < R ? rB / g : -1;
-  uint32_t qa[8][4];
-  {
-    const uint16_t* qA = a.q_new + ((static_cast<size_t>(b) * f + max(iA, 0)) * c.Hq + h * g + rA % g) * kHeadDim;
-    const uint16_t* qB = a.q_new + ((static_cast<size_t>(b) * f + max(iB, 0)) * c.Hq + h * g + rB % g) * kHeadDim;
-#pragma unroll
-    for (int ks = 0; ks < 8; ++ks) {
-      const int d0 = 16 * ks + 2 * (lane & 3);
-      qa[ks][0] = iA >= 0 ? *reinterpret_cast<const uint32_t*>(qA + d0) : 0u;
-      qa[ks][1] = iB >= 0 ? *reinterpret_cast<const uint32_t*>(qB + d0) : 0u;
-      qa[ks][2] = iA >= 0 ? *reinterpret_cast<const uint32_t*>(qA + d0 + 8) : 0u;
-      qa[ks][3] = iB >= 0 ? *reinterpret_cast<const uint32_t*>(qB + d0 + 8) : 0u;
-    }
+  // Q tile: rows row0 .. row0 + 128 MT - 1, zero for padding rows
+  for (int e = tid; e < MT * kMTile * 16; e += kThreads) {
+    const int row = e >> 4, ch = e & 15;
+    const int rr = row0 + row, i = rr >> 3, j = rr & 7;
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (!bad && i < f && j < g)
+      v = *reinterpret_cast<const uint4*>(a.q_new + ((static_cast<size_t>(b) * f + i) * c.Hq + h * g + j) * kHeadDim +
+                                          ch * 8);
+    *reinterpret_cast<uint4*>(smem + kOffQ + (ch >> 3) * kQHalf + sw128(row, ch & 7)) = v;
   }
+  fence_proxy_async_smem();
+  __syncthreads();
 
-  float mA = kNegInf, mB = kNegInf, lA = 0.f, lB = 0.f;
-  float o[16][4];
+  if (warp == 0) {
+    // ------------------------------------------------------- producer ---
+    for (int t = 0; t < n_tiles; ++t) {
+      const int st = t % kStages;
+      if (t >= kStages && !warp_wait(bar(kBarKvEmpty + st), ((t / kStages) - 1) & 1)) {
+        if (lane == 0) record_error(c.status, RESA_DEV_WAIT_TIMEOUT, bh);
+        break;
+      }
+      uint8_t* kst = smem + kOffKV + st * kStageBytes;
+      const uint32_t kdst = sbase + kOffKV + st * kStageBytes;
+      if (t < n_pref) {
+        if (lane == 0) {
+          const int kb = (t0 + t) * kTileKeys;
+          int rows[4], pages = 0;
+          for (int pg = 0; pg < 4; ++pg) {
+            rows[pg] = -1;
+            const int blk = kb / kBlock + pg;
+            if (blk * kBlock >= P) continue;
+            const int page = c.page_table[static_cast<size_t>(b) * c.max_blocks + blk];
+            if (page < 0 || page >= c.num_pages) {
+              record_error(c.status, RESA_DEV_PAGE_RANGE, b);
+              continue;
+            }
+            rows[pg] = (page * c.Hkv + h) * kBlock;
+            ++pages;
+          }
+          mbar_arrive_expect_tx(bar(kBarKvFull + st), pages * 4 * 2048);
+          for (int pg = 0; pg < 4; ++pg) {
+            if (rows[pg] < 0) continue;
+            const uint32_t o = pg * 2048;
+            tma_load_2d(kdst + o, &tm_k, bar(kBarKvFull + st), 0, rows[pg]);
+            tma_load_2d(kdst + kKVHalf + o, &tm_k, bar(kBarKvFull + st), 64, rows[pg]);
+            tma_load_2d(kdst + 2 * kKVHalf + o, &tm_v, bar(kBarKvFull + st), 0, rows[pg]);
+            tma_load_2d(kdst + 3 * kKVHalf + o, &tm_v, bar(kBarKvFull + st), 64, rows[pg]);
+          }
+        }
+      } else {
+        const int tb = (t - n_pref) * kTileKeys;  // tail tile: tokens tb .. tb + 63 of the f
+        for (int e = lane; e < kTileKeys * 16; e += 32) {
+          const int row = e >> 4, ch = e & 15, tok = tb + row;
+          uint4 kv = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
+          if (tok < f) {
+            const size_t src = ((static_cast<size_t>(b) * f + tok) * c.Hkv + h) * kHeadDim + ch * 8;
+            kv = *reinterpret_cast<const uint4*>(a.k_new + src);
+            vv = *reinterpret_cast<const uint4*>(a.v_new + src);
+          }
+          const uint32_t off = (ch >> 3) * kKVHalf + sw128(row, ch & 7);
+          *reinterpret_cast<uint4*>(kst + off) = kv;
+          *reinterpret_cast<uint4*>(kst + 2 * kKVHalf + off) = vv;
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(kBarKvFull + st));
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA ---
+    if (lane == 0) {
+      auto issue_pv = [&](int u) -> bool {
+        const int bu = u & 1, su = u % kStages;
+        if (!mbar_wait_bounded(bar(kBarPFull + bu), (u >> 1) & 1)) return false;
+        tc_fence_after();
+        const uint32_t vbase = sbase + kOffKV + su * kStageBytes + 2 * kKVHalf;
+        for (int mt = 0; mt < MT; ++mt) {
+          const uint32_t pbase = sbase + kOffP + (bu * kMaxMTiles + mt) * kPTile;
+          for (int kk = 0; kk < kTileKeys / 16; ++kk)
+            umma_bf16(tmem + kColO + mt * 128, smem_desc_sw128(pbase + kk * 32, 16, 1024),
+                      smem_desc_sw128(vbase + kk * 2048, kKVHalf, 1024), kIdescO, (u > 0 || kk > 0) ? 1u : 0u);
+        }
+        umma_commit(bar(kBarODone + bu));
+        umma_commit(bar(kBarKvEmpty + su));
+        return true;
+      };
+      bool ok = true;
+      for (int t = 0; t < n_tiles && ok; ++t) {
+        const int st = t % kStages, buf = t & 1;
+        if (!mbar_wait_bounded(bar(kBarKvFull + st), (t / kStages) & 1)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t kbase = sbase + kOffKV + st * kStageBytes;
+        for (int mt = 0; mt < MT; ++mt) {
+          for (int ks = 0; ks < 8; ++ks) {
+            const uint32_t half = ks >> 2, off = (ks & 3) * 32;
+            umma_bf16(tmem + kColS + (buf * kMaxMTiles + mt) * kTileKeys,
+                      smem_desc_sw128(sbase + kOffQ + half * kQHalf + mt * kPTile + off, 16, 1024),
+                      smem_desc_sw128(kbase + half * kKVHalf + off, 16, 1024), kIdescS, ks > 0 ? 1u : 0u);
+          }
+        }
+        umma_commit(bar(kBarSFull + buf));
+        if (t >= 1) ok = issue_pv(t - 1);
+      }
+      if (ok && n_tiles > 0) ok = issue_pv(n_tiles - 1);
+      if (!ok) record_error(c.status, RESA_DEV_WAIT_TIMEOUT, bh);
+      // let every issued MMA finish before the CTA may free its TMEM
+      umma_commit(bar(kBarFinal));
+      mbar_wait_bounded(bar(kBarFinal), 0);
+    }
+    __syncwarp();
+  } else if (warp >= kSoftmaxWarp0) {
+    // -------------------------------------------------------- softmax ---
+    const int mt = (warp - kSoftmaxWarp0) >> 2, quarter = warp & 3;
+    const int rit = quarter * 32 + lane;  // row within the M-tile = TMEM lane
+    const int rr = row0 + mt * kMTile + rit;
+    const int ti = rr >> 3, tj = rr & 7;
+    const bool valid_row = ti < f && tj < g;
+    const int sm_tid = (warp - kSoftmaxWarp0) * 32 + lane;  // 0 .. 128 MT - 1
+    if (mt < MT) {
+      const uint32_t lane_base = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+      float m_used = kNegInf, l = 0.f;
+      bool ok = true;
+      for (int t = 0; t < n_tiles; ++t) {
+        const int buf = t & 1, st = t % kStages;
+        if (!warp_wait(bar(kBarSFull + buf), (t >> 1) & 1)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        float sv[kTileKeys];
+        {
+          uint32_t r[32];
+          const uint32_t col = kColS + (buf * kMaxMTiles + mt) * kTileKeys;
+          tmem_ld32(lane_base + col, r);
+          tmem_ld_wait();
 #pragma unroll
-  for (int nt = 0; nt < 16; ++nt) o[nt][0] = o[nt][1] = o[nt][2] = o[nt][3] = 0.f;
-
-  // One 64-key tile held in stage `st`. Key column c is visible to row r iff
-  // visible(c, i(r)): prefix tiles: kb + c < P; tail tiles: tb + c < f && tb + c <= i.
-  auto tile = [&](int st, bool tail, int kbase) {
-    const uint32_t kst = sbase + st * kStageBytes, vst = kst + 2 * kHalfBytes;
-    float sc[8][4];
+          for (int x = 0; x < 32; ++x) sv[x] = __uint_as_float(r[x]);
+          tmem_ld32(lane_base + col + 32, r);
+          tmem_ld_wait();
 #pragma unroll
-    for (int nt = 0; nt < 8; ++nt) sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
-    {
-      const int j = lane >> 3, r = lane & 7;
+          for (int x = 0; x < 32; ++x) sv[32 + x] = __uint_as_float(r[x]);
+        }
+        const bool tail = t >= n_pref;
+        const int kb = tail ? (t - n_pref) * kTileKeys : (t0 + t) * kTileKeys;
+        const int lim = tail ? min(f - 1 - kb, ti - kb) : P - 1 - kb;  // key c visible iff c <= lim
+        float mx = kNegInf;
 #pragma unroll
-      for (int ks = 0; ks < 8; ++ks) {
-        const int chunk = 2 * ks + (j & 1);
+        for (int x = 0; x < kTileKeys; ++x) {
+          sv[x] = (x <= lim) ? sv[x] * a.scale_log2 : kNegInf;
+          mx = fmaxf(mx, sv[x]);
+        }
+        // P[buf] is reused every second tile: PV of tile t - 2 must be done
+        if (t >= 2 && !warp_wait(bar(kBarODone + buf), ((t - 2) >> 1) & 1)) {
+          ok = false;
+          break;
+        }
+        const float m_new = fmaxf(m_used, mx);
+        const bool need = m_new > m_used + kRescaleLog2;  // per row
+        const bool scale_o = need && t >= 1 && m_used != kNegInf;
+        // The O rescale is warp-collective (tcgen05.ld/st are .sync.aligned):
+        // the whole warp takes it if any of its rows needs it; rows that do
+        // not keep alpha = 1.
+        if (__any_sync(0xffffffffu, scale_o)) {
+          // O row *= 2^(m_used - m_new) once PV of tile t - 1 has landed
+          if (!warp_wait(bar(kBarODone + ((t - 1) & 1)), ((t - 1) >> 1) & 1)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const float alpha = scale_o ? exp2f(m_used - m_new) : 1.f;
+          for (int ch = 0; ch < 4; ++ch) {
+            uint32_t r[32];
+            tmem_ld32(lane_base + kColO + mt * 128 + ch * 32, r);
+            tmem_ld_wait();
 #pragma unroll
-        for (int np = 0; np < 4; ++np) {
-          const int key = 16 * np + r + 8 * (j >> 1);
-          uint32_t b0, b1, b2, b3;
-          ldsm_x4(kst + (chunk >> 3) * kHalfBytes + sw128(key, chunk & 7), b0, b1, b2, b3);
-          mma_bf16_16816(sc[2 * np], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], b0, b1);
-          mma_bf16_16816(sc[2 * np + 1], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], b2, b3);
+            for (int x = 0; x < 32; ++x) r[x] = __float_as_uint(__uint_as_float(r[x]) * alpha);
+            tmem_st32(lane_base + kColO + mt * 128 + ch * 32, r);
+          }
+          tmem_st_wait();
+          l *= alpha;
+        }
+        if (need) m_used = m_new;
+        const float base = safe_base(m_used);
+        uint8_t* prow = smem + kOffP + (buf * kMaxMTiles + mt) * kPTile;
+#pragma unroll
+        for (int ch = 0; ch < 8; ++ch) {
+          uint32_t w[4];
+#pragma unroll
+          for (int x = 0; x < 4; ++x) {
+            w[x] = pack_bf16x2(exp2f(sv[8 * ch + 2 * x] - base), exp2f(sv[8 * ch + 2 * x + 1] - base));
+            l += bf16_lo(w[x]) + bf16_hi(w[x]);
+          }
+          *reinterpret_cast<uint4*>(prow + sw128(rit, ch)) = make_uint4(w[0], w[1], w[2], w[3]);
+        }
+        if (!tail && kb + kTileKeys > P) {
+          // keys past the prefix may sit in unwritten memory: zero their V rows
+          uint8_t* v = smem + kOffKV + st * kStageBytes + 2 * kKVHalf;
+          const int first = max(0, P - kb);
+          for (int e = sm_tid; e < (kTileKeys - first) * 16; e += kMTile * MT) {
+            const int row = first + (e >> 4), hf = (e >> 3) & 1;
+            *reinterpret_cast<uint4*>(v + hf * kKVHalf + row * 128 + (e & 7) * 16) = make_uint4(0, 0, 0, 0);
+          }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        mbar_arrive(bar(kBarPFull + buf));
+      }
+      if (!ok && lane == 0) record_error(c.status, RESA_DEV_WAIT_TIMEOUT, bh);
+      // ---- epilogue: normalised partial O and log2-sum-exp of this row ----
+      const bool have = ok && n_tiles > 0 &&
+                        warp_wait(bar(kBarODone + ((n_tiles - 1) & 1)), ((n_tiles - 1) >> 1) & 1);
+      if (have) tc_fence_after();
+      const float inv = (have && l > 0.f) ? 1.f / l : 0.f;
+      const size_t prow_g = (static_cast<size_t>(b) * f + ti) * c.Hq + h * g + tj;
+      float* dst = a.o_part + (prow_g * a.splits + s) * kHeadDim;
+      for (int ch = 0; ch < 4; ++ch) {
+        uint32_t r[32];
+        if (have) {
+          tmem_ld32(lane_base + kColO + mt * 128 + ch * 32, r);
+          tmem_ld_wait();
+        }
+        if (valid_row && !bad) {
+#pragma unroll
+          for (int x = 0; x < 32; x += 4)
+            *reinterpret_cast<float4*>(dst + ch * 32 + x) =
+                have ? make_float4(__uint_as_float(r[x]) * inv, __uint_as_float(r[x + 1]) * inv,
+                                   __uint_as_float(r[x + 2]) * inv, __uint_as_float(r[x + 3]) * inv)
+                     : make_float4(0.f, 0.f, 0.f, 0.f);
         }
       }
-    }
-    float tmA = kNegInf, tmB = kNegInf;
-#pragma unroll
-    for (int nt = 0; nt < 8; ++nt) {
-#pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        const int col = kbase + 8 * nt + 2 * (lane & 3) + e;
-        const bool vA = tail ? (col < f && col <= iA) : (col < P);
-        const bool vB = tail ? (col < f && col <= iB) : (col < P);
-        sc[nt][e] = vA ? sc[nt][e] * a.scale_log2 : kNegInf;
-        sc[nt][2 + e] = vB ? sc[nt][2 + e] * a.scale_log2 : kNegInf;
-        tmA = fmaxf(tmA, sc[nt][e]);
-        tmB = fmaxf(tmB, sc[nt][2 + e]);
-      }
-    }
-#pragma unroll
-    for (int x = 1; x < 4; x <<= 1) {
-      tmA = fmaxf(tmA, __shfl_xor_sync(0xffffffffu, tmA, x));
-      tmB = fmaxf(tmB, __shfl_xor_sync(0xffffffffu, tmB, x));
-    }
-    const float nA = fmaxf(mA, tmA), nB = fmaxf(mB, tmB);
-    const float baseA = safe_base(nA), baseB = safe_base(nB);
-    const float alA = exp2f(mA - baseA), alB = exp2f(mB - baseB);
-    mA = nA;
-    mB = nB;
-    uint32_t pa[4][4];
-    float sumA = 0.f, sumB = 0.f;
-#pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-#pragma unroll
-      for (int hf = 0; hf < 2; ++hf) {
-        const int nt = 2 * kk + hf;
-        const uint32_t xa = pack_bf16x2(exp2f(sc[nt][0] - baseA), exp2f(sc[nt][1] - baseA));
-        const uint32_t xb = pack_bf16x2(exp2f(sc[nt][2] - baseB), exp2f(sc[nt][3] - baseB));
-        sumA += bf16_lo(xa) + bf16_hi(xa);
-        sumB += bf16_lo(xb) + bf16_hi(xb);
-        pa[kk][2 * hf] = xa;
-        pa[kk][2 * hf + 1] = xb;
-      }
-    }
-    lA = lA * alA + sumA;
-    lB = lB * alB + sumB;
-#pragma unroll
-    for (int nt = 0; nt < 16; ++nt) {
-      o[nt][0] *= alA;
-      o[nt][1] *= alA;
-      o[nt][2] *= alB;
-      o[nt][3] *= alB;
-    }
-    {
-      const int j = lane >> 3, r = lane & 7;
-#pragma unroll
-      for (int kk = 0; kk < 4; ++kk) {
-        const int key = 16 * kk + r + 8 * (j & 1);
-#pragma unroll
-        for (int dp = 0; dp < 8; ++dp) {
-          const int chunk = 2 * dp + (j >> 1);
-          uint32_t b0, b1, b2, b3;
-          ldsm_x4_t(vst + (chunk >> 3) * kHalfBytes + sw128(key, chunk & 7), b0, b1, b2, b3);
-          mma_bf16_16816(o[2 * dp], pa[kk][0], pa[kk][1], pa[kk][2], pa[kk][3], b0, b1);
-          mma_bf16_16816(o[2 * dp + 1], pa[kk][0], pa[kk][1], pa[kk][2], pa[kk][3], b2, b3);
-        }
-      }
-    }
-  };
-
-  bool failed = false;
-  int lt = 0;
-  for (; lt < n_pref; ++lt) {
-    const int st = lt % kStages;
-    const uint32_t par = (lt / kStages) & 1;
-    if (tid == 0) sh_ok = mbar_wait_bounded(bar0 + 8 * st, par) ? 1 : 0;
-    __syncthreads();
-    if (!sh_ok) {
-      failed = true;
-      break;
-    }
-    mbar_try_wait(bar0 + 8 * st, par);
-    const int kb = (t0 + lt) * kTile;
-    if (kb + kTile > P) {  // last prefix tile: zero V rows past the prefix (unwritten memory may be NaN)
-      uint8_t* v = smem + st * kStageBytes + 2 * kHalfBytes;
-      for (int e = tid; e < kTile * 16; e += kWarps * 32) {
-        const int row = e >> 4, hf = (e >> 3) & 1;
-        if (kb + row >= P) *reinterpret_cast<uint4*>(v + hf * kHalfBytes + row * 128 + (e & 7) * 16) =
-                               make_uint4(0, 0, 0, 0);
-      }
-      __syncthreads();
-    }
-    tile(st, false, kb);
-    __syncthreads();
-    if (tid == 0 && lt + kStages < n_pref) {
-      fence_proxy_async_smem();
-      issue(lt + kStages, st);
+      if (valid_row && !bad) a.lse_part[prow_g * a.splits + s] = (have && l > 0.f) ? m_used + log2f(l) : kNegInf;
     }
   }
-  if (failed) {
-    if (tid == 0) {
-      record_error(c.status, RESA_DEV_WAIT_TIMEOUT, bh);
-      for (int k = lt; k < min(n_pref, lt + kStages); ++k)
-        mbar_wait_bounded(bar0 + 8 * (k % kStages), (k / kStages) & 1);
-    }
-    return;
-  }
-  // causal tail from k_new / v_new (written into stage 0 with the TMA layout)
-  for (int tt = 0; tt < n_tail; ++tt) {
-    const int tb = tt * kTile;
-    uint8_t* kst = smem;
-    uint8_t* vst = smem + 2 * kHalfBytes;
-    for (int e = tid; e < kTile * 16; e += kWarps * 32) {
-      const int row = e >> 4, ch = e & 15;
-      const int t = tb + row;
-      uint4 kv = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
-      if (t < f) {
-        const size_t src = ((static_cast<size_t>(b) * f + t) * c.Hkv + h) * kHeadDim + ch * 8;
-        kv = *reinterpret_cast<const uint4*>(a.k_new + src);
-        vv = *reinterpret_cast<const uint4*>(a.v_new + src);
-      }
-      const uint32_t off = (ch >> 3) * kHalfBytes + sw128(row, ch & 7);
-      *reinterpret_cast<uint4*>(kst + off) = kv;
-      *reinterpret_cast<uint4*>(vst + off) = vv;
-    }
-    __syncthreads();
-    tile(0, true, tb);
-    __syncthreads();
-  }
-
-  // epilogue: normalised partial O and log2-sum-exp per row
-#pragma unroll
-  for (int x = 1; x < 4; x <<= 1) {
-    lA += __shfl_xor_sync(0xffffffffu, lA, x);
-    lB += __shfl_xor_sync(0xffffffffu, lB, x);
-  }
-  const float invA = lA > 0.f ? 1.f / lA : 0.f, invB = lB > 0.f ? 1.f / lB : 0.f;
-#pragma unroll
-  for (int hf = 0; hf < 2; ++hf) {
-    const int r = hf ? rB : rA;
-    const int i = hf ? iB : iA;
-    if (i < 0) continue;
-    const size_t prow = (static_cast<size_t>(b) * f + i) * c.Hq + h * g + r % g;
-    float* dst = a.o_part + (prow * a.splits + s) * kHeadDim;
-    const float inv = hf ? invB : invA;
-#pragma unroll
-    for (int nt = 0; nt < 16; ++nt) {
-      const int d = 8 * nt + 2 * (lane & 3);
-      *reinterpret_cast<float2*>(dst + d) = make_float2(o[nt][2 * hf] * inv, o[nt][2 * hf + 1] * inv);
-    }
-    if ((lane & 3) == 0) {
-      const float l = hf ? lB : lA, m = hf ? mB : mA;
-      a.lse_part[prow * a.splits + s] = l > 0.f ? m + log2f(l) : kNegInf;
-    }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
   }
 }
 
 }  // namespace
 
-int rectify_row_groups(int g, int f) { return (g * f + kRows - 1) / kRows; }
+int rectify_row_groups(int g, int f) {
+  (void)g;
+  return (8 * f + kRowsPerCta - 1) / kRowsPerCta;
+}
 
 cudaError_t launch_rectify(const CacheView& c, const CUtensorMap& tm_k, const CUtensorMap& tm_v,
                            const uint16_t* q_new, const uint16_t* k_new, const uint16_t* v_new, int f,
@@ -313,7 +395,7 @@ cudaError_t launch_rectify(const CacheView& c, const CUtensorMap& tm_k, const CU
   if (e != cudaSuccess) return e;
   RectArgs a{q_new, k_new, v_new, f, splits, sm_scale * 1.44269504088896340736f, o_part, lse_part};
   const dim3 grid(splits, rectify_row_groups(c.g, f), c.B * c.Hkv);
-  return launch_pdl(rectify_kernel, grid, dim3(kWarps * 32), kSmem, st, tm_k, tm_v, c, a);
+  return launch_pdl(rectify_kernel, grid, dim3(kThreads), kSmem, st, tm_k, tm_v, c, a);
 }
 
 }  // namespace resa

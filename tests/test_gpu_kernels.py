@@ -270,6 +270,32 @@ def test_rectify_matches_oracle(g, Hkv, lens, f):
         assert np.allclose(lse[b], l, atol=2e-3, rtol=0)
 
 
+@pytest.mark.parametrize("f,T", [(32, 3000), (16, 1500), (64, 1200)])
+def test_rectify_rescale_path(f, T):
+    """Keys whose magnitude ramps up along the positions (and log-normal
+    outlier channels) make row maxima grow tile after tile, at different
+    tiles for different rows, exercising the tensor-memory O rescale."""
+    g, Hkv = 7, 2
+    gr = synth.rng(90 + f)
+    ramp = (1.0 + 6.0 * np.arange(T) / T)[None, :, None]
+    chan = np.exp(0.7 * gr.standard_normal((Hkv, 1, 128)))
+    Kf = gr.standard_normal((Hkv, T, 128)) * ramp * chan
+    K = synth.f32_to_bf16_bits(Kf.astype(np.float32))
+    V = synth.normal_bf16(gr, (Hkv, T, 128))
+    cache = H.make_cache([K], [V], g * Hkv, (T + 15) // 16 + 2)
+    qn = synth.normal_bf16(gr, (1, f, g * Hkv, 128))
+    kn = np.ascontiguousarray(np.transpose(K[:, T - f:], (1, 0, 2)))[None]
+    vn = np.ascontiguousarray(np.transpose(V[:, T - f:], (1, 0, 2)))[None]
+    out = torch.empty((1, f, g * Hkv, 128), dtype=torch.bfloat16, device="cuda")
+    ws, nb = H.workspace(cache, 8, 0, f)
+    resa.resa_rectify_attention(cache.struct, H.dev_bf16(qn), H.dev_bf16(kn), H.dev_bf16(vn), f,
+                                resa.params(0.1, 0, 0), out, None, ws, nb)
+    assert resa.resa_read_device_error(cache.struct) == (0, 0)
+    o, _ = O.rectify_attention(O.widen_bf16(qn[0]), O.widen_bf16(K), O.widen_bf16(V), O.widen_bf16(kn[0]),
+                               O.widen_bf16(vn[0]), T, 1 / math.sqrt(128))
+    H.check_outputs(H.host_f64(out)[0], o, "rectify with growing maxima")
+
+
 def test_rectify_too_short_sequence_is_reported():
     Ks, Vs = seq_inputs(40, 1, 1, [8])
     cache = H.make_cache(Ks, Vs, 4, 4)
