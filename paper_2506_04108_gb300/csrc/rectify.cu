@@ -15,7 +15,7 @@
 // CTA = 12 warps:
 //   warp 0      TMA producer: 64-key K and V tiles of the prefix, one
 //               SWIZZLE_128B box per 16-key page per 64-column half, into a
-//               2-stage ring (kv_full / kv_empty mbarriers); the causal tail
+//               3-stage ring (kv_full / kv_empty mbarriers); the causal tail
 //               is written by the warp's lanes in the same swizzled layout.
 //   warp 1      allocates 512 TMEM columns; lane 0 issues the MMAs:
 //               S[t] = Q K^T (M 128, N 64, K 128; both operands K-major) into
@@ -40,7 +40,7 @@ constexpr int kMTile = 128;
 constexpr int kMaxMTiles = 2;
 constexpr int kRowsPerCta = kMTile * kMaxMTiles;  // 256
 constexpr int kTileKeys = 64;
-constexpr int kStages = 2;
+constexpr int kStages = 3;
 constexpr int kQHalf = kRowsPerCta * 128;          // [256 rows][64 dims] bf16 = 32 KB
 constexpr int kKVHalf = kTileKeys * 128;           // [64 keys][64 dims] = 8 KB
 constexpr int kStageBytes = 4 * kKVHalf;           // K (2 halves) + V (2 halves) = 32 KB
@@ -48,7 +48,7 @@ constexpr int kPTile = kMTile * 128;               // [128 rows][64 keys] = 16 K
 constexpr int kOffQ = 0;
 constexpr int kOffP = 2 * kQHalf;                  // 64 KB
 constexpr int kOffKV = kOffP + 2 * kMaxMTiles * kPTile;   // 128 KB
-constexpr int kOffBar = kOffKV + kStages * kStageBytes;  // 192 KB
+constexpr int kOffBar = kOffKV + kStages * kStageBytes;  // 224 KB
 constexpr int kSmem = kOffBar + 256 + 1024;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColO = 0;
@@ -59,7 +59,9 @@ constexpr float kRescaleLog2 = 8.f;
 constexpr float kNegInf = -__builtin_huge_valf();
 
 // barrier slots (uint64) in the barrier region
-constexpr int kBarKvFull = 0, kBarKvEmpty = 2, kBarSFull = 4, kBarPFull = 6, kBarODone = 8, kBarFinal = 10;
+constexpr int kBarKvFull = 0, kBarKvEmpty = kStages, kBarSFull = 2 * kStages, kBarPFull = kBarSFull + 2,
+              kBarODone = kBarPFull + 2, kBarFinal = kBarODone + 2;
+static_assert(8 * (kBarFinal + 1) <= 128, "barriers overlap the TMEM address slot");
 
 struct RectArgs {
   const uint16_t* q_new;  // [B][f][Hq][128]
@@ -103,9 +105,11 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
   const int MT = min(kMaxMTiles, (rows_total - row0 + kMTile - 1) / kMTile);
 
   if (tid == 0) {
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < kStages; ++i) {
       mbar_init(bar(kBarKvFull + i), 1);
       mbar_init(bar(kBarKvEmpty + i), 1);
+    }
+    for (int i = 0; i < 2; ++i) {
       mbar_init(bar(kBarSFull + i), 1);
       mbar_init(bar(kBarPFull + i), kMTile * MT);
       mbar_init(bar(kBarODone + i), 1);
@@ -269,27 +273,37 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
           break;
         }
         tc_fence_after();
-        float sv[kTileKeys];
+        float sv[kTileKeys];  // raw scores q.k of this row
         {
-          uint32_t r[32];
+          uint32_t r0[32], r1[32];
           const uint32_t col = kColS + (buf * kMaxMTiles + mt) * kTileKeys;
-          tmem_ld32(lane_base + col, r);
+          tmem_ld32(lane_base + col, r0);
+          tmem_ld32(lane_base + col + 32, r1);
           tmem_ld_wait();
 #pragma unroll
-          for (int x = 0; x < 32; ++x) sv[x] = __uint_as_float(r[x]);
-          tmem_ld32(lane_base + col + 32, r);
-          tmem_ld_wait();
-#pragma unroll
-          for (int x = 0; x < 32; ++x) sv[32 + x] = __uint_as_float(r[x]);
+          for (int x = 0; x < 32; ++x) {
+            sv[x] = __uint_as_float(r0[x]);
+            sv[32 + x] = __uint_as_float(r1[x]);
+          }
         }
         const bool tail = t >= n_pref;
         const int kb = tail ? (t - n_pref) * kTileKeys : (t0 + t) * kTileKeys;
         const int lim = tail ? min(f - 1 - kb, ti - kb) : P - 1 - kb;  // key c visible iff c <= lim
-        float mx = kNegInf;
+        if (lim < kTileKeys - 1) {
 #pragma unroll
-        for (int x = 0; x < kTileKeys; ++x) {
-          sv[x] = (x <= lim) ? sv[x] * a.scale_log2 : kNegInf;
-          mx = fmaxf(mx, sv[x]);
+          for (int x = 0; x < kTileKeys; ++x) sv[x] = (x <= lim) ? sv[x] : kNegInf;
+        }
+        float mx;
+        {
+          float m4[4];
+#pragma unroll
+          for (int y = 0; y < 4; ++y) {
+            float v = sv[y];
+#pragma unroll
+            for (int x = y + 4; x < kTileKeys; x += 4) v = fmaxf(v, sv[x]);
+            m4[y] = v;
+          }
+          mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * a.scale_log2;  // scale > 0 keeps the order
         }
         // P[buf] is reused every second tile: PV of tile t - 2 must be done
         if (t >= 2 && !warp_wait(bar(kBarODone + buf), ((t - 2) >> 1) & 1)) {
@@ -322,18 +336,22 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
           l *= alpha;
         }
         if (need) m_used = m_new;
-        const float base = safe_base(m_used);
+        const float nbase = -safe_base(m_used);
         uint8_t* prow = smem + kOffP + (buf * kMaxMTiles + mt) * kPTile;
+        float ls = 0.f;
 #pragma unroll
         for (int ch = 0; ch < 8; ++ch) {
           uint32_t w[4];
 #pragma unroll
           for (int x = 0; x < 4; ++x) {
-            w[x] = pack_bf16x2(exp2f(sv[8 * ch + 2 * x] - base), exp2f(sv[8 * ch + 2 * x + 1] - base));
-            l += bf16_lo(w[x]) + bf16_hi(w[x]);
+            const float p0 = ex2_approx(fmaf(sv[8 * ch + 2 * x], a.scale_log2, nbase));
+            const float p1 = ex2_approx(fmaf(sv[8 * ch + 2 * x + 1], a.scale_log2, nbase));
+            ls += p0 + p1;
+            w[x] = pack_bf16x2(p0, p1);
           }
           *reinterpret_cast<uint4*>(prow + sw128(rit, ch)) = make_uint4(w[0], w[1], w[2], w[3]);
         }
+        l += ls;
         if (!tail && kb + kTileKeys > P) {
           // keys past the prefix may sit in unwritten memory: zero their V rows
           uint8_t* v = smem + kOffKV + st * kStageBytes + 2 * kKVHalf;

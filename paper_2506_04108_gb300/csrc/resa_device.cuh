@@ -31,6 +31,13 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// 2^x on the special-function unit (PTX ex2.approx, flush-to-zero): -inf -> 0.
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // --------------------------------------------- programmatic dependent launch ---
 // Every kernel is launched with programmatic stream serialization: it lets the
 // next kernel on the stream start launching (launch_dependents), and waits for
