@@ -30,7 +30,8 @@
  *     out) are recorded in cache->device_status (first error wins) and the
  *     affected work is skipped; resa_read_device_error() returns them.
  *   - Supported geometry: head_dim 128, block_size 16, GQA group size
- *     num_q_heads / num_kv_heads in [1, 8]; other values return
+ *     num_q_heads / num_kv_heads in [1, 8], batch <= 1024, and
+ *     max_blocks_per_seq <= 409600 (6.5M tokens); other values return
  *     RESA_ERR_UNSUPPORTED.
  *   - The library is stateless apart from per-device cached attributes and is
  *     safe to call from several host threads; calls that share buffers must

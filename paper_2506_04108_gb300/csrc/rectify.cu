@@ -15,7 +15,7 @@
 // CTA = 12 warps:
 //   warp 0      TMA producer: 64-key K and V tiles of the prefix, one
 //               SWIZZLE_128B box per 16-key page per 64-column half, into a
-//               3-stage ring (kv_full / kv_empty mbarriers); the causal tail
+//               4-stage ring (kv_full / kv_empty mbarriers); the causal tail
 //               is written by the warp's lanes in the same swizzled layout.
 //   warp 1      allocates 512 TMEM columns; lane 0 issues the MMAs:
 //               S[t] = Q K^T (M 128, N 64, K 128; both operands K-major) into
@@ -23,7 +23,9 @@
 //               P K-major from shared memory, V MN-major) into TMEM O.
 //   warps 4-11  softmax: one thread per query row (TMEM lane), so the row max
 //               and sum need no shuffles. P is written to shared memory as
-//               bf16. O is rescaled in TMEM only when a row maximum grows by
+//               bf16 (one buffer: a tile's P is written at the end of its
+//               softmax, once the previous tile's PV has completed). O is
+//               rescaled in TMEM only when a row maximum grows by
 //               more than 2^8 (exact: the exponent base is carried along).
 // TMEM columns: O[mt] = [128 mt, 128 mt + 128), S[buf][mt] = 256 + 64 (2 buf + mt).
 // Every mbarrier wait is bounded; a wait that runs out records
@@ -40,14 +42,14 @@ constexpr int kMTile = 128;
 constexpr int kMaxMTiles = 2;
 constexpr int kRowsPerCta = kMTile * kMaxMTiles;  // 256
 constexpr int kTileKeys = 64;
-constexpr int kStages = 3;
+constexpr int kStages = 4;
 constexpr int kQHalf = kRowsPerCta * 128;          // [256 rows][64 dims] bf16 = 32 KB
 constexpr int kKVHalf = kTileKeys * 128;           // [64 keys][64 dims] = 8 KB
 constexpr int kStageBytes = 4 * kKVHalf;           // K (2 halves) + V (2 halves) = 32 KB
 constexpr int kPTile = kMTile * 128;               // [128 rows][64 keys] = 16 KB
 constexpr int kOffQ = 0;
 constexpr int kOffP = 2 * kQHalf;                  // 64 KB
-constexpr int kOffKV = kOffP + 2 * kMaxMTiles * kPTile;   // 128 KB
+constexpr int kOffKV = kOffP + kMaxMTiles * kPTile;      // 96 KB (one P buffer per M-tile)
 constexpr int kOffBar = kOffKV + kStages * kStageBytes;  // 224 KB
 constexpr int kSmem = kOffBar + 256 + 1024;
 constexpr uint32_t kTmemCols = 512;
@@ -142,14 +144,25 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
   if (bad && tid == 0 && s == 0 && rg == 0) record_error(c.status, RESA_DEV_SEQ_LEN_RANGE, b);
 
   // Q tile: rows row0 .. row0 + 128 MT - 1, zero for padding rows
-  for (int e = tid; e < MT * kMTile * 16; e += kThreads) {
-    const int row = e >> 4, ch = e & 15;
-    const int rr = row0 + row, i = rr >> 3, j = rr & 7;
-    uint4 v = make_uint4(0, 0, 0, 0);
-    if (!bad && i < f && j < g)
-      v = *reinterpret_cast<const uint4*>(a.q_new + ((static_cast<size_t>(b) * f + i) * c.Hq + h * g + j) * kHeadDim +
-                                          ch * 8);
-    *reinterpret_cast<uint4*>(smem + kOffQ + (ch >> 3) * kQHalf + sw128(row, ch & 7)) = v;
+  for (int e0 = 0; e0 < MT * kMTile * 16; e0 += 4 * kThreads) {  // four loads in flight per thread
+    uint4 v[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int e = e0 + u * kThreads + tid;
+      const int row = e >> 4, ch = e & 15;
+      const int rr = row0 + row, i = rr >> 3, j = rr & 7;
+      v[u] = make_uint4(0, 0, 0, 0);
+      if (e < MT * kMTile * 16 && !bad && i < f && j < g)
+        v[u] = *reinterpret_cast<const uint4*>(a.q_new + ((static_cast<size_t>(b) * f + i) * c.Hq + h * g + j) *
+                                                             kHeadDim + ch * 8);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int e = e0 + u * kThreads + tid;
+      const int row = e >> 4, ch = e & 15;
+      if (e < MT * kMTile * 16)
+        *reinterpret_cast<uint4*>(smem + kOffQ + (ch >> 3) * kQHalf + sw128(row, ch & 7)) = v[u];
+    }
   }
   fence_proxy_async_smem();
   __syncthreads();
@@ -218,7 +231,7 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
         tc_fence_after();
         const uint32_t vbase = sbase + kOffKV + su * kStageBytes + 2 * kKVHalf;
         for (int mt = 0; mt < MT; ++mt) {
-          const uint32_t pbase = sbase + kOffP + (bu * kMaxMTiles + mt) * kPTile;
+          const uint32_t pbase = sbase + kOffP + mt * kPTile;
           for (int kk = 0; kk < kTileKeys / 16; ++kk)
             umma_bf16(tmem + kColO + mt * 128, smem_desc_sw128(pbase + kk * 32, 16, 1024),
                       smem_desc_sw128(vbase + kk * 2048, kKVHalf, 1024), kIdescO, (u > 0 || kk > 0) ? 1u : 0u);
@@ -305,8 +318,8 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
           }
           mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * a.scale_log2;  // scale > 0 keeps the order
         }
-        // P[buf] is reused every second tile: PV of tile t - 2 must be done
-        if (t >= 2 && !warp_wait(bar(kBarODone + buf), ((t - 2) >> 1) & 1)) {
+        // P is single-buffered: PV of tile t - 1 must have consumed it
+        if (t >= 1 && !warp_wait(bar(kBarODone + ((t - 1) & 1)), ((t - 1) >> 1) & 1)) {
           ok = false;
           break;
         }
@@ -317,11 +330,7 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
         // the whole warp takes it if any of its rows needs it; rows that do
         // not keep alpha = 1.
         if (__any_sync(0xffffffffu, scale_o)) {
-          // O row *= 2^(m_used - m_new) once PV of tile t - 1 has landed
-          if (!warp_wait(bar(kBarODone + ((t - 1) & 1)), ((t - 1) >> 1) & 1)) {
-            ok = false;
-            break;
-          }
+          // O row *= 2^(m_used - m_new); PV of tile t - 1 has landed (waited above)
           tc_fence_after();
           const float alpha = scale_o ? exp2f(m_used - m_new) : 1.f;
           for (int ch = 0; ch < 4; ++ch) {
@@ -337,7 +346,7 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
         }
         if (need) m_used = m_new;
         const float nbase = -safe_base(m_used);
-        uint8_t* prow = smem + kOffP + (buf * kMaxMTiles + mt) * kPTile;
+        uint8_t* prow = smem + kOffP + mt * kPTile;
         float ls = 0.f;
 #pragma unroll
         for (int ch = 0; ch < 8; ++ch) {

@@ -92,6 +92,7 @@ resa_status_t check_cache(const resa_cache_t* c) {
   if (static_cast<int64_t>(c->num_pages) * c->num_kv_heads * c->block_size > INT32_MAX) return RESA_ERR_UNSUPPORTED;
   if (static_cast<int64_t>(c->max_blocks_per_seq) * c->block_size > INT32_MAX / 2) return RESA_ERR_UNSUPPORTED;
   if (c->max_blocks_per_seq > select_max_blocks()) return RESA_ERR_UNSUPPORTED;
+  if (c->batch > 1024) return RESA_ERR_UNSUPPORTED;
   if (c->k_pool == nullptr || c->v_pool == nullptr || c->page_table == nullptr || c->seq_lens == nullptr ||
       c->summaries == nullptr || c->device_status == nullptr)
     return RESA_ERR_INVALID_ARG;

@@ -1,10 +1,10 @@
 // Block selection (Section 2.1 "Block Selection"; Eq. 4 and Eq. 5).
 //
-// score_kernel  grid (block chunks, KV head, sequence). Each CTA forms the
-//               pooled query of its GQA group (mean of the g heads, fp32) and
-//               scores 64 blocks: a half-warp takes one block, each lane one
-//               16-byte chunk (8 dims) of k_min and k_max, so a warp reads two
-//               contiguous 512-byte summaries per load instruction. The
+// score_kernel  persistent, one CTA per SM: streams the block summaries in
+//               32 KB chunks with bulk copies through a shared-memory ring and
+//               scores them with the pooled query of the chunk's GQA group
+//               (mean of the g heads, fp32); a half-warp takes one block, a
+//               lane one 16-byte piece (8 dims) of k_min and k_max, and the
 //               128-dim sum is a fixed-order butterfly over the 16 lanes.
 // topn_kernel   one 8-CTA cluster per (sequence, KV head). The n of Eq. 5 is
 //               evaluated on the device from the device-resident length. The
@@ -26,8 +26,6 @@ namespace resa {
 namespace {
 
 constexpr int kScoreWarps = 8;
-constexpr int kScoreUnroll = 4;                                    // 2 blocks per warp per step
-constexpr int kBlocksPerScoreCta = kScoreWarps * 2 * kScoreUnroll;  // 64
 constexpr int kTopnCluster = 8;                                   // CTAs per (sequence, KV head)
 constexpr int kTopnThreads = 256;
 constexpr int kTopnWarps = kTopnThreads / 32;
@@ -45,82 +43,160 @@ __device__ __forceinline__ float quest_term8(const float* q, const uint4& mn, co
   return s;
 }
 
-// Loads of one CTA iteration: 8 warps x 2 half-warps x kScoreUnroll blocks.
-struct SummaryChunk {
-  uint4 mn[kScoreUnroll], mx[kScoreUnroll];
-};
+// Persistent score kernel: one CTA per SM. The (sequence, KV head) units'
+// summaries are cut into chunks of 64 blocks (32 KB, contiguous); CTA x owns
+// the chunk range [x * per, (x + 1) * per) of the flattened chunk list.
+// Thread 0 streams the chunks with 1-D bulk copies into a kScoreStages-deep
+// shared-memory ring; the 8 warps score each chunk from shared memory (a
+// half-warp per block, a lane per 16-byte piece of k_min and k_max, fixed
+// order 16-lane reduction) and release the stage.
+constexpr int kScoreStages = 6;
+constexpr int kMaxBatch = 1024;  // sequences per call supported by the score kernel
+constexpr int kChunkBlocks = 64;
+constexpr int kChunkBytes = kChunkBlocks * 2 * kHeadDim * 2;  // 32 KB
+constexpr int kScoreSmem = kScoreStages * kChunkBytes + 1024 + 2 * kScoreStages * 8 + 64;
 
-__device__ __forceinline__ void load_chunk(SummaryChunk& r, const uint16_t* sb, int base, int end, int warp,
-                                           int half, int ch) {
-#pragma unroll
-  for (int u = 0; u < kScoreUnroll; ++u) {
-    const int blk = base + warp * (2 * kScoreUnroll) + 2 * u + half;
-    if (blk < end) {
-      const uint16_t* s = sb + static_cast<size_t>(blk) * 2 * kHeadDim + ch * 8;
-      r.mn[u] = *reinterpret_cast<const uint4*>(s);
-      r.mx[u] = *reinterpret_cast<const uint4*>(s + kHeadDim);
-    } else {
-      r.mn[u] = make_uint4(0, 0, 0, 0);
-      r.mx[u] = make_uint4(0, 0, 0, 0);
+__global__ void __launch_bounds__(256, 1) score_kernel(CacheView c, const uint16_t* __restrict__ q,
+                                                       float* __restrict__ scores) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const uint32_t sbase = smem_u32(smem);
+  const uint32_t full0 = sbase + kScoreStages * kChunkBytes;
+  const uint32_t empty0 = full0 + 8 * kScoreStages;
+  // per-sequence block counts and the chunk prefix over (sequence, head) units
+  __shared__ int sh_M[kMaxBatch];
+  __shared__ int sh_pref[kMaxBatch + 1];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if (tid == 0) {
+    for (int i = 0; i < kScoreStages; ++i) {
+      mbar_init(full0 + 8 * i, 1);
+      mbar_init(empty0 + 8 * i, kScoreWarps);
     }
+    fence_mbar_init();
   }
-}
-
-// Grid (chunks, KV head, sequence) sized to one wave; CTA x scores the blocks
-// [x * per, min(M, (x + 1) * per)) of its (sequence, head), per = ceil(M /
-// chunks), 64 blocks per iteration. The next iteration's summaries are
-// loaded before the current one is reduced, and the first loads are issued
-// before the group's queries are read.
-__global__ void __launch_bounds__(256) score_kernel(CacheView c, const uint16_t* __restrict__ q,
-                                                    float* __restrict__ scores, int chunks) {
   pdl_launch_dependents();
   pdl_wait();
-  const int b = blockIdx.z, h = blockIdx.y;
-  const int T = c.seq_lens[b];
-  if (T < 0 || T > c.max_blocks * kBlock) return;  // reported by topn_kernel
-  const int M = (T + kBlock - 1) / kBlock;
-  const int per = (M + chunks - 1) / chunks;
-  const int start = blockIdx.x * per, end = min(M, start + per);
-  if (start >= end) return;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int ch = lane & 15, half = lane >> 4;
-  const uint16_t* sb = c.summ + (static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks * 2 * kHeadDim;
-  SummaryChunk cur, nxt;
-  load_chunk(cur, sb, start, end, warp, half, ch);
-
-  // pooled query (mean of the group's heads) for this lane's 8 dims
-  float qp[8];
-#pragma unroll
-  for (int j = 0; j < 8; ++j) qp[j] = 0.f;
-  const uint16_t* qg = q + (static_cast<size_t>(b) * c.Hq + h * c.g) * kHeadDim + ch * 8;
-  for (int i = 0; i < c.g; ++i) {
-    const uint4 v = *reinterpret_cast<const uint4*>(qg + i * kHeadDim);
-    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      qp[2 * j] += bf16_lo(w[j]);
-      qp[2 * j + 1] += bf16_hi(w[j]);
-    }
+  for (int b = tid; b < c.B; b += blockDim.x) {
+    const int T = c.seq_lens[b];
+    sh_M[b] = (T < 0 || T > c.max_blocks * kBlock) ? 0 : (T + kBlock - 1) / kBlock;  // bad lengths: top-n reports
   }
-  const float inv_g = 1.0f / static_cast<float>(c.g);
+  __syncthreads();
+  if (warp == 0) {  // exclusive prefix of Hkv * chunks-per-head over sequences
+    int carry = 0;
+    for (int b0 = 0; b0 < c.B; b0 += 32) {
+      const int b = b0 + lane;
+      const int v = b < c.B ? c.Hkv * ((sh_M[b] + kChunkBlocks - 1) / kChunkBlocks) : 0;
+      int x = v;
 #pragma unroll
-  for (int j = 0; j < 8; ++j) qp[j] = qp[j] * inv_g;
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+      }
+      if (b < c.B) sh_pref[b] = carry + x - v;
+      carry += __shfl_sync(0xffffffffu, x, 31);
+    }
+    if (lane == 0) sh_pref[c.B] = carry;
+  }
+  __syncthreads();
+  const int total = sh_pref[c.B];
+  const int per = (total + gridDim.x - 1) / gridDim.x;
+  const int c0 = blockIdx.x * per, c1 = min(total, c0 + per);
+  const int nmine = max(0, c1 - c0);
 
-  float* out = scores + (static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks;
-  for (int base = start; base < end; base += kBlocksPerScoreCta) {
-    const bool more = base + kBlocksPerScoreCta < end;
-    if (more) load_chunk(nxt, sb, base + kBlocksPerScoreCta, end, warp, half, ch);
+  // chunk index -> (sequence, head, first block, blocks): binary search of the prefix
+  auto locate = [&](int ci, int& b, int& h, int& blk0, int& nblk) {
+    int lo = 0, hi = c.B - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (sh_pref[mid] <= ci) lo = mid;
+      else hi = mid - 1;
+    }
+    b = lo;
+    const int M = sh_M[b];
+    const int per_head = (M + kChunkBlocks - 1) / kChunkBlocks;
+    const int r = ci - sh_pref[b];
+    h = r / per_head;
+    blk0 = (r % per_head) * kChunkBlocks;
+    nblk = min(kChunkBlocks, M - blk0);
+  };
+  auto issue = [&](int k) {  // thread 0: my k-th chunk into stage k % kScoreStages
+    int b, h, blk0, nblk;
+    locate(c0 + k, b, h, blk0, nblk);
+    const uint32_t bar = full0 + 8 * (k % kScoreStages);
+    const uint32_t bytes = static_cast<uint32_t>(nblk) * 2 * kHeadDim * 2;
+    mbar_arrive_expect_tx(bar, bytes);
+    bulk_load(sbase + (k % kScoreStages) * kChunkBytes,
+              c.summ + ((static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks + blk0) * 2 * kHeadDim, bytes, bar);
+  };
+  if (tid == 0)
+    for (int k = 0; k < min(kScoreStages, nmine); ++k) issue(k);
+
+  const int ch = lane & 15, half = lane >> 4;
+  int cur_unit = -1;
+  float qp[8];
+  for (int k = 0; k < nmine; ++k) {
+    const int st = k % kScoreStages;
+    int b, h, blk0, nblk;
+    locate(c0 + k, b, h, blk0, nblk);
+    const int unit = b * c.Hkv + h;
+    if (unit != cur_unit) {  // pooled query (mean of the group's heads), this lane's 8 dims
+      cur_unit = unit;
 #pragma unroll
-    for (int u = 0; u < kScoreUnroll; ++u) {
-      const int blk = base + warp * (2 * kScoreUnroll) + 2 * u + half;
-      float sc = quest_term8(qp, cur.mn[u], cur.mx[u]);
+      for (int j = 0; j < 8; ++j) qp[j] = 0.f;
+      const uint16_t* qg = q + (static_cast<size_t>(b) * c.Hq + h * c.g) * kHeadDim + ch * 8;
+      uint4 qv[kMaxGroup];  // all g rows in flight at once (g <= 8)
+#pragma unroll
+      for (int i = 0; i < kMaxGroup; ++i)
+        qv[i] = i < c.g ? *reinterpret_cast<const uint4*>(qg + i * kHeadDim) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+      for (int i = 0; i < kMaxGroup; ++i) {
+        const uint32_t w[4] = {qv[i].x, qv[i].y, qv[i].z, qv[i].w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          qp[2 * j] += bf16_lo(w[j]);
+          qp[2 * j + 1] += bf16_hi(w[j]);
+        }
+      }
+      const float inv_g = 1.0f / static_cast<float>(c.g);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) qp[j] = qp[j] * inv_g;
+    }
+    int ok = 1;
+    if (lane == 0) ok = mbar_wait_bounded(full0 + 8 * st, (k / kScoreStages) & 1) ? 1 : 0;
+    ok = __shfl_sync(0xffffffffu, ok, 0);
+    if (!ok) {
+      if (lane == 0) record_error(c.status, RESA_DEV_WAIT_TIMEOUT, unit);
+      break;
+    }
+    mbar_try_wait(full0 + 8 * st, (k / kScoreStages) & 1);
+    const uint8_t* chunk = smem + st * kChunkBytes;
+    float* out = scores + static_cast<size_t>(unit) * c.max_blocks + blk0;
+#pragma unroll
+    for (int u = 0; u < kChunkBlocks / (2 * kScoreWarps); ++u) {
+      const int blk = warp * (kChunkBlocks / kScoreWarps) + 2 * u + half;
+      float sc = 0.f;
+      if (blk < nblk) {
+        const uint4 mn = *reinterpret_cast<const uint4*>(chunk + blk * 512 + ch * 16);
+        const uint4 mx = *reinterpret_cast<const uint4*>(chunk + blk * 512 + 256 + ch * 16);
+        sc = quest_term8(qp, mn, mx);
+      }
       sc += __shfl_xor_sync(0xffffffffu, sc, 8);
       sc += __shfl_xor_sync(0xffffffffu, sc, 4);
       sc += __shfl_xor_sync(0xffffffffu, sc, 2);
       sc += __shfl_xor_sync(0xffffffffu, sc, 1);
-      if (ch == 0 && blk < end) out[blk] = sc;
+      if (ch == 0 && blk < nblk) out[blk] = sc;
     }
-    if (more) cur = nxt;
+    __syncwarp();
+    if (lane == 0) mbar_arrive(empty0 + 8 * st);
+    if (tid == 0 && k + kScoreStages < nmine) {
+      // every warp has released this stage before it is refilled
+      if (!mbar_wait_bounded(empty0 + 8 * st, (k / kScoreStages) & 1)) {
+        record_error(c.status, RESA_DEV_WAIT_TIMEOUT, unit);
+      } else {
+        fence_proxy_async_smem();
+        issue(k + kScoreStages);
+      }
+    }
   }
 }
 
@@ -197,7 +273,19 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
   const int lo = rank * per, cnt = max(0, min(M, lo + per) - lo);
   const float* sc = scores + (static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks + lo;
   const int first_forced = M - n_local - lo;
-  for (int i = tid; i < cnt; i += kTopnThreads) keys[i] = (i >= first_forced) ? 0xFFFFFFFFu : score_key(sc[i]);
+  for (int i0 = 0; i0 < cnt; i0 += 4 * kTopnThreads) {  // four loads in flight per thread
+    float v[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int i = i0 + u * kTopnThreads + tid;
+      v[u] = i < cnt ? sc[i] : 0.f;
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int i = i0 + u * kTopnThreads + tid;
+      if (i < cnt) keys[i] = (i >= first_forced) ? 0xFFFFFFFFu : score_key(v[u]);
+    }
+  }
   const int cnt_round = (cnt + 31) / 32 * 32;
 
   // ---- radix select of the n-th largest key across the cluster ----
@@ -347,22 +435,12 @@ int select_max_blocks() { return kTopnCluster * (kTopnSmemMax / static_cast<int>
 cudaError_t launch_select(const CacheView& c, const uint16_t* q, double keep, int n_min, int n_local,
                           int32_t* indices, int32_t* counts, int n_cap, float* scores, int sm_count,
                           cudaStream_t st) {
-  // one wave of resident score CTAs, shared by batch * KV heads
-  static std::atomic<int> occ_cache{0};
-  int occ = occ_cache.load(std::memory_order_relaxed);
-  if (occ == 0) {
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, score_kernel, kScoreWarps * 32, 0) != cudaSuccess ||
-        occ < 1)
-      occ = 1;
-    occ_cache.store(occ, std::memory_order_relaxed);
-  }
-  const int units = c.B * c.Hkv;
-  const int max_chunks = (c.max_blocks + kBlocksPerScoreCta - 1) / kBlocksPerScoreCta;
-  int chunks = occ * sm_count / units;
-  if (chunks > max_chunks) chunks = max_chunks;
-  if (chunks < 1) chunks = 1;
-  cudaError_t e = launch_pdl(score_kernel, dim3(chunks, c.Hkv, c.B), dim3(kScoreWarps * 32), 0, st, c, q, scores,
-                             chunks);
+  cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(score_kernel), kScoreSmem, 3);
+  if (e != cudaSuccess) return e;
+  // one persistent CTA per SM (never more than the chunks there can be)
+  const int max_chunks = c.B * c.Hkv * ((c.max_blocks + kChunkBlocks - 1) / kChunkBlocks);
+  const int grid = max(1, min(sm_count, max_chunks));
+  e = launch_pdl(score_kernel, dim3(grid), dim3(kScoreWarps * 32), kScoreSmem, st, c, q, scores);
   if (e != cudaSuccess) return e;
   const size_t smem = select_smem_bytes(c.max_blocks);
   if (smem > 48 * 1024) {
