@@ -225,16 +225,21 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA ---
     if (lane == 0) {
+      // Base descriptors; an MMA's operand is base + (byte offset >> 4) (the
+      // 14-bit start-address field cannot carry: shared memory is < 256 KB).
+      const uint64_t dq = smem_desc_sw128(sbase + kOffQ, 16, 1024);
+      const uint64_t dp = smem_desc_sw128(sbase + kOffP, 16, 1024);
+      const uint64_t dkv = smem_desc_sw128(sbase + kOffKV, 16, 1024);
+      const uint64_t dvv = smem_desc_sw128(sbase + kOffKV + 2 * kKVHalf, kKVHalf, 1024);
       auto issue_pv = [&](int u) -> bool {
         const int bu = u & 1, su = u % kStages;
         if (!mbar_wait_bounded(bar(kBarPFull + bu), (u >> 1) & 1)) return false;
         tc_fence_after();
-        const uint32_t vbase = sbase + kOffKV + su * kStageBytes + 2 * kKVHalf;
+        const uint64_t dv = dvv + ((su * kStageBytes) >> 4);
         for (int mt = 0; mt < MT; ++mt) {
-          const uint32_t pbase = sbase + kOffP + mt * kPTile;
           for (int kk = 0; kk < kTileKeys / 16; ++kk)
-            umma_bf16(tmem + kColO + mt * 128, smem_desc_sw128(pbase + kk * 32, 16, 1024),
-                      smem_desc_sw128(vbase + kk * 2048, kKVHalf, 1024), kIdescO, (u > 0 || kk > 0) ? 1u : 0u);
+            umma_bf16(tmem + kColO + mt * 128, dp + ((mt * kPTile + kk * 32) >> 4), dv + ((kk * 2048) >> 4), kIdescO,
+                      (u > 0 || kk > 0) ? 1u : 0u);
         }
         umma_commit(bar(kBarODone + bu));
         umma_commit(bar(kBarKvEmpty + su));
@@ -248,13 +253,13 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
           break;
         }
         tc_fence_after();
-        const uint32_t kbase = sbase + kOffKV + st * kStageBytes;
+        const uint64_t dk = dkv + ((st * kStageBytes) >> 4);
         for (int mt = 0; mt < MT; ++mt) {
           for (int ks = 0; ks < 8; ++ks) {
-            const uint32_t half = ks >> 2, off = (ks & 3) * 32;
+            const uint32_t off = (ks & 3) * 32;
             umma_bf16(tmem + kColS + (buf * kMaxMTiles + mt) * kTileKeys,
-                      smem_desc_sw128(sbase + kOffQ + half * kQHalf + mt * kPTile + off, 16, 1024),
-                      smem_desc_sw128(kbase + half * kKVHalf + off, 16, 1024), kIdescS, ks > 0 ? 1u : 0u);
+                      dq + (((ks >> 2) * kQHalf + mt * kPTile + off) >> 4),
+                      dk + (((ks >> 2) * kKVHalf + off) >> 4), kIdescS, ks > 0 ? 1u : 0u);
           }
         }
         umma_commit(bar(kBarSFull + buf));

@@ -2,10 +2,10 @@
 // combine of split partials (Algorithm 2, "Combine").
 //
 // sparse_decode_kernel, grid (splits, KV head, sequence), 4 warps:
-//   * The CTA owns selected blocks [s*per, min(n, (s+1)*per)) of its
-//     (sequence, KV head), per = ceil(n / splits). Warp w takes every 4th of
-//     them, so the group's g <= 8 query heads share every K/V block fetched
-//     (GQA-shared fetch).
+//   * The CTA owns index slots [s*per, (s+1)*per) of its (sequence, KV head),
+//     per = ceil(n_cap / splits), and attends to the selected blocks among
+//     them (slots below counts[b][h]). Warp w takes every 4th, so the group's
+//     g <= 8 query heads share every K/V block fetched (GQA-shared fetch).
 //   * Each warp streams its blocks through a private 3-stage shared-memory
 //     ring: lane 0 issues four bulk-tensor TMA copies per block (K and V, two
 //     64-column halves each, SWIZZLE_128B) that complete on the stage's
@@ -67,8 +67,16 @@ __global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid
   __syncwarp();
   pdl_launch_dependents();
   pdl_wait();
+  // Splits cover the index capacity [0, n_cap): the CTA's id range is known
+  // before `counts` arrives, so ids, length, count and queries load together.
+  const int per = (a.n_cap + a.splits - 1) / a.splits;
+  const int j0 = s * per;
+  const int nj_cap = max(0, min(a.n_cap, j0 + per) - j0);
+  const int cnt_cap = nj_cap > warp ? (nj_cap - warp + kWarps - 1) / kWarps : 0;
+  const int32_t* idx = a.indices + static_cast<size_t>(b * c.Hkv + h) * a.n_cap + j0 + warp;
   const int T = c.seq_lens[b];
   int n = a.counts[b * c.Hkv + h];
+  int pre_blk = lane < cnt_cap ? idx[lane * kWarps] : -1;
   if (T < 0 || T > c.max_blocks * kBlock) {
     if (threadIdx.x == 0 && s == 0) record_error(c.status, RESA_DEV_SEQ_LEN_RANGE, b);
     n = 0;
@@ -77,29 +85,25 @@ __global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid
     n = 0;
   }
   const int M = (max(T, 0) + kBlock - 1) / kBlock;
-  const int per = (n + a.splits - 1) / a.splits;
-  const int j0 = s * per;
-  const int nj = max(0, min(n, j0 + per) - j0);
-  const int cnt = nj > warp ? (nj - warp + kWarps - 1) / kWarps : 0;
-  const int32_t* idx = a.indices + static_cast<size_t>(b * c.Hkv + h) * a.n_cap + j0 + warp;
+  // this warp's blocks are ids j0 + warp + kWarps * it < n
+  const int cnt = max(0, min(cnt_cap, (n - j0 - warp + kWarps - 1) / kWarps));
 
-  // Block id and page of the warp's it-th block; the first 32 are resolved by
-  // all lanes at once (two round trips), later ones on demand. page = -1: the
-  // block id is out of range; -2: its page is. Such blocks are fully masked.
-  auto resolve = [&](int it, int& blk) -> int {
-    blk = idx[it * kWarps];
+  // Page of block blk, or -1 if the id is out of range, -2 if its page is.
+  // Such blocks are fully masked (and reported).
+  auto page_of = [&](int blk) -> int {
     if (blk < 0 || blk >= M) return -1;
     const int page = c.page_table[static_cast<size_t>(b) * c.max_blocks + blk];
     return (page >= 0 && page < c.num_pages) ? page : -2;
   };
-  int pre_blk = -1, pre_page = -1;
-  if (lane < cnt) pre_page = resolve(lane, pre_blk);
-  auto info = [&](int it, int& blk) -> int {  // warp-uniform
+  int pre_page = -1;
+  if (lane < cnt) pre_page = page_of(pre_blk);
+  auto info = [&](int it, int& blk) -> int {  // warp-uniform; ids beyond 32 per warp load on demand
     if (it < 32) {
       blk = __shfl_sync(0xffffffffu, pre_blk, it);
       return __shfl_sync(0xffffffffu, pre_page, it);
     }
-    return resolve(it, blk);
+    blk = idx[it * kWarps];
+    return page_of(blk);
   };
   auto issue = [&](int it, int st) {  // warp-uniform; lane 0 issues
     int blk;
