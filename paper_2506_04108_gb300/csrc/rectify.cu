@@ -15,19 +15,21 @@
 // CTA = 12 warps:
 //   warp 0      TMA producer: 64-key K and V tiles of the prefix, one
 //               SWIZZLE_128B box per 16-key page per 64-column half, into a
-//               4-stage ring (kv_full / kv_empty mbarriers); the causal tail
+//               5-stage ring (kv_full / kv_empty mbarriers); the causal tail
 //               is written by the warp's lanes in the same swizzled layout.
 //   warp 1      allocates 512 TMEM columns; lane 0 issues the MMAs:
-//               S[t] = Q K^T (M 128, N 64, K 128; both operands K-major) into
-//               a double-buffered TMEM S, and O += P V (M 128, N 128, K 64;
-//               P K-major from shared memory, V MN-major) into TMEM O.
+//               S[t] = Q K^T (M 128, N 64, K 128; both operands K-major from
+//               shared memory) into a double-buffered TMEM S, and
+//               O += P V (M 128, N 128, K 64) with P read from tensor memory
+//               (the A operand) and V an MN-major shared-memory operand.
 //   warps 4-11  softmax: one thread per query row (TMEM lane), so the row max
-//               and sum need no shuffles. P is written to shared memory as
-//               bf16 (one buffer: a tile's P is written at the end of its
-//               softmax, once the previous tile's PV has completed). O is
-//               rescaled in TMEM only when a row maximum grows by
-//               more than 2^8 (exact: the exponent base is carried along).
-// TMEM columns: O[mt] = [128 mt, 128 mt + 128), S[buf][mt] = 256 + 64 (2 buf + mt).
+//               and sum need no shuffles. P (bf16, key pairs packed per
+//               column) is stored over the first 32 columns of its own S tile,
+//               so no shared memory or wait on the previous PV is needed; S of
+//               tile t + 2 is issued only after PV of tile t has read that P.
+//               O is rescaled in TMEM only when a row maximum grows by more
+//               than 2^8 (exact: the exponent base is carried along).
+// TMEM columns: O[mt] = [128 mt, 128 mt + 128), S/P[buf][mt] = 256 + 64 (2 buf + mt).
 // Every mbarrier wait is bounded; a wait that runs out records
 // RESA_DEV_WAIT_TIMEOUT and the CTA winds down, freeing its TMEM.
 #include "resa_device.cuh"
@@ -42,14 +44,13 @@ constexpr int kMTile = 128;
 constexpr int kMaxMTiles = 2;
 constexpr int kRowsPerCta = kMTile * kMaxMTiles;  // 256
 constexpr int kTileKeys = 64;
-constexpr int kStages = 4;
+constexpr int kStages = 5;
 constexpr int kQHalf = kRowsPerCta * 128;          // [256 rows][64 dims] bf16 = 32 KB
 constexpr int kKVHalf = kTileKeys * 128;           // [64 keys][64 dims] = 8 KB
 constexpr int kStageBytes = 4 * kKVHalf;           // K (2 halves) + V (2 halves) = 32 KB
-constexpr int kPTile = kMTile * 128;               // [128 rows][64 keys] = 16 KB
+constexpr int kQTile = kMTile * 128;               // one M-tile of one Q half = 16 KB
 constexpr int kOffQ = 0;
-constexpr int kOffP = 2 * kQHalf;                  // 64 KB
-constexpr int kOffKV = kOffP + kMaxMTiles * kPTile;      // 96 KB (one P buffer per M-tile)
+constexpr int kOffKV = 2 * kQHalf;                       // 64 KB
 constexpr int kOffBar = kOffKV + kStages * kStageBytes;  // 224 KB
 constexpr int kSmem = kOffBar + 256 + 1024;
 constexpr uint32_t kTmemCols = 512;
@@ -63,7 +64,8 @@ constexpr float kNegInf = -__builtin_huge_valf();
 // barrier slots (uint64) in the barrier region
 constexpr int kBarKvFull = 0, kBarKvEmpty = kStages, kBarSFull = 2 * kStages, kBarPFull = kBarSFull + 2,
               kBarODone = kBarPFull + 2, kBarFinal = kBarODone + 2;
-static_assert(8 * (kBarFinal + 1) <= 128, "barriers overlap the TMEM address slot");
+constexpr int kTmemSlot = 240;  // byte offset of the TMEM base address in the barrier region
+static_assert(8 * (kBarFinal + 1) <= kTmemSlot, "barriers overlap the TMEM address slot");
 
 struct RectArgs {
   const uint16_t* q_new;  // [B][f][Hq][128]
@@ -96,7 +98,7 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
   const uint32_t sbase = smem_u32(smem);
   const uint32_t bar0 = sbase + kOffBar;
   auto bar = [&](int slot) -> uint32_t { return bar0 + 8u * slot; };
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kOffBar + 128);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kOffBar + kTmemSlot);
 
   const int s = blockIdx.x, rg = blockIdx.y, bh = blockIdx.z;
   const int b = bh / c.Hkv, h = bh % c.Hkv;
@@ -228,7 +230,6 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
       // Base descriptors; an MMA's operand is base + (byte offset >> 4) (the
       // 14-bit start-address field cannot carry: shared memory is < 256 KB).
       const uint64_t dq = smem_desc_sw128(sbase + kOffQ, 16, 1024);
-      const uint64_t dp = smem_desc_sw128(sbase + kOffP, 16, 1024);
       const uint64_t dkv = smem_desc_sw128(sbase + kOffKV, 16, 1024);
       const uint64_t dvv = smem_desc_sw128(sbase + kOffKV + 2 * kKVHalf, kKVHalf, 1024);
       auto issue_pv = [&](int u) -> bool {
@@ -237,9 +238,11 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
         tc_fence_after();
         const uint64_t dv = dvv + ((su * kStageBytes) >> 4);
         for (int mt = 0; mt < MT; ++mt) {
+          // P of (u, mt) sits in the first 32 columns of S[bu][mt], 8 columns per 16 keys
+          const uint32_t ptmem = tmem + kColS + (bu * kMaxMTiles + mt) * kTileKeys;
           for (int kk = 0; kk < kTileKeys / 16; ++kk)
-            umma_bf16(tmem + kColO + mt * 128, dp + ((mt * kPTile + kk * 32) >> 4), dv + ((kk * 2048) >> 4), kIdescO,
-                      (u > 0 || kk > 0) ? 1u : 0u);
+            umma_bf16_tmem_a(tmem + kColO + mt * 128, ptmem + kk * 8, dv + ((kk * 2048) >> 4), kIdescO,
+                             (u > 0 || kk > 0) ? 1u : 0u);
         }
         umma_commit(bar(kBarODone + bu));
         umma_commit(bar(kBarKvEmpty + su));
@@ -252,13 +255,18 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
           ok = false;
           break;
         }
+        // S(t) overwrites S[buf], whose first columns hold P(t - 2): PV(t - 2) must be done
+        if (t >= 2 && !mbar_wait_bounded(bar(kBarODone + buf), ((t - 2) >> 1) & 1)) {
+          ok = false;
+          break;
+        }
         tc_fence_after();
         const uint64_t dk = dkv + ((st * kStageBytes) >> 4);
         for (int mt = 0; mt < MT; ++mt) {
           for (int ks = 0; ks < 8; ++ks) {
             const uint32_t off = (ks & 3) * 32;
             umma_bf16(tmem + kColS + (buf * kMaxMTiles + mt) * kTileKeys,
-                      dq + (((ks >> 2) * kQHalf + mt * kPTile + off) >> 4),
+                      dq + (((ks >> 2) * kQHalf + mt * kQTile + off) >> 4),
                       dk + (((ks >> 2) * kKVHalf + off) >> 4), kIdescS, ks > 0 ? 1u : 0u);
           }
         }
@@ -323,19 +331,17 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
           }
           mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * a.scale_log2;  // scale > 0 keeps the order
         }
-        // P is single-buffered: PV of tile t - 1 must have consumed it
-        if (t >= 1 && !warp_wait(bar(kBarODone + ((t - 1) & 1)), ((t - 1) >> 1) & 1)) {
-          ok = false;
-          break;
-        }
         const float m_new = fmaxf(m_used, mx);
         const bool need = m_new > m_used + kRescaleLog2;  // per row
         const bool scale_o = need && t >= 1 && m_used != kNegInf;
         // The O rescale is warp-collective (tcgen05.ld/st are .sync.aligned):
-        // the whole warp takes it if any of its rows needs it; rows that do
-        // not keep alpha = 1.
+        // the whole warp takes it if any of its rows needs it (rows that do
+        // not keep alpha = 1), once PV of tile t - 1 has landed.
         if (__any_sync(0xffffffffu, scale_o)) {
-          // O row *= 2^(m_used - m_new); PV of tile t - 1 has landed (waited above)
+          if (!warp_wait(bar(kBarODone + ((t - 1) & 1)), ((t - 1) >> 1) & 1)) {
+            ok = false;
+            break;
+          }
           tc_fence_after();
           const float alpha = scale_o ? exp2f(m_used - m_new) : 1.f;
           for (int ch = 0; ch < 4; ++ch) {
@@ -351,21 +357,19 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
         }
         if (need) m_used = m_new;
         const float nbase = -safe_base(m_used);
-        uint8_t* prow = smem + kOffP + mt * kPTile;
-        float ls = 0.f;
+        uint32_t w[kTileKeys / 2];  // P row as packed bf16 pairs (keys 2x, 2x + 1)
+        float ls[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int ch = 0; ch < 8; ++ch) {
-          uint32_t w[4];
-#pragma unroll
-          for (int x = 0; x < 4; ++x) {
-            const float p0 = ex2_approx(fmaf(sv[8 * ch + 2 * x], a.scale_log2, nbase));
-            const float p1 = ex2_approx(fmaf(sv[8 * ch + 2 * x + 1], a.scale_log2, nbase));
-            ls += p0 + p1;
-            w[x] = pack_bf16x2(p0, p1);
-          }
-          *reinterpret_cast<uint4*>(prow + sw128(rit, ch)) = make_uint4(w[0], w[1], w[2], w[3]);
+        for (int x = 0; x < kTileKeys / 2; ++x) {
+          const float p0 = ex2_approx(fmaf(sv[2 * x], a.scale_log2, nbase));
+          const float p1 = ex2_approx(fmaf(sv[2 * x + 1], a.scale_log2, nbase));
+          ls[x & 3] += p0 + p1;
+          w[x] = pack_bf16x2(p0, p1);
         }
-        l += ls;
+        l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+        // P over the S columns it came from (this thread's lane; S is in registers)
+        tmem_st32(lane_base + kColS + (buf * kMaxMTiles + mt) * kTileKeys, w);
+        tmem_st_wait();
         if (!tail && kb + kTileKeys > P) {
           // keys past the prefix may sit in unwritten memory: zero their V rows
           uint8_t* v = smem + kOffKV + st * kStageBytes + 2 * kKVHalf;
@@ -374,8 +378,8 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
             const int row = first + (e >> 4), hf = (e >> 3) & 1;
             *reinterpret_cast<uint4*>(v + hf * kKVHalf + row * 128 + (e & 7) * 16) = make_uint4(0, 0, 0, 0);
           }
+          fence_proxy_async_smem();  // generic stores, read next by the tensor core
         }
-        fence_proxy_async_smem();
         tc_fence_before();
         mbar_arrive(bar(kBarPFull + buf));
       }
