@@ -111,18 +111,19 @@ def source_hash(*names) -> str:
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(kernel: str, workload: str, src_hash: str):
-    """DRAM bytes per launch of `kernel` from a committed ncu summary, if its
-    recorded source hash still matches the kernel source; else None."""
+def profiled_traffic(call: str, workload: str, src_hash: str):
+    """DRAM bytes per call of type `call` (summed over the call's kernels) from
+    a committed ncu summary, if its recorded source hash still matches the
+    kernel source; else None."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(path):
         return None
     with open(path) as fh:
         table = json.load(fh)
-    e = table.get(kernel, {}).get(workload)
+    e = table.get(call, {}).get(workload)
     if not e or e.get("source_hash") != src_hash:
         return None
-    return e.get("dram_bytes_per_launch")
+    return e.get("dram_bytes_per_call")
 
 
 class ClockSampler:
@@ -541,13 +542,15 @@ def run_ours(args, w: synth.Workload):
     calls["rectify"]["frac_bf16_sustained"] = round(rflops / (mean_us["rectify"] * 1e-6) / 1e12 /
                                                     float(peaks["bf16_tflops_sustained"]), 3)
     dominant = max(per_step_us, key=per_step_us.get)
-    kernel, src = {"decode": ("sparse_decode_kernel", "sparse_decode.cu"), "select": ("topn_kernel", "select.cu"),
-                   "rectify": ("rectify_kernel", "rectify.cu"), "commit": ("commit_append_kernel", "kv_commit.cu"),
+    kernel, src = {"decode": ("sparse_decode_kernel+merge_kernel", "sparse_decode.cu"),
+                   "select": ("score_kernel+topn_kernel", "select.cu"),
+                   "rectify": ("rectify_kernel+merge_kernel", "rectify.cu"),
+                   "commit": ("commit_append_kernel", "kv_commit.cu"),
                    "overwrite": ("commit_overwrite_kernel", "kv_commit.cu")}[dominant]
     achieved = algo[dominant] / (mean_us[dominant] * 1e-6) / 1e9
     roofline = {"bound": "hbm", "call": dominant, "kernel": kernel, "achieved": round(achieved, 1), "peak": hbm,
                 "unit": "GB/s", "frac": round(achieved / hbm, 3), "peak_kind": peak_kind,
-                "traffic": profiled_traffic(kernel, w.name, source_hash(src)),
+                "traffic": profiled_traffic(dominant, w.name, source_hash(src)),
                 "algorithmic_bytes_per_launch": int(algo[dominant]),
                 "timing": "CUDA events around a graph of the step's calls of this kind; per call = total / calls"}
 
@@ -615,6 +618,82 @@ def run_e2e(args, layers, graph):
                     "CUDA graph), device -> pinned host copies of every decode and rectify output"}
 
 
+def run_rectify_sweep(args):
+    """Rectification-only sweep (the f x context grid): per cell, dense causal
+    attention of f new queries (28 q / 4 KV heads, d 128, batch 1) against a
+    cached context T, then the K/V overwrite and block-summary refresh of the
+    touched blocks. Enough independent caches rotate per cell that the
+    rotation's working set exceeds L2. One JSON line per cell."""
+    import torch
+    from paper_2506_04108_gb300 import build as _b
+    from paper_2506_04108_gb300 import resa
+    _b.build()
+    resa.load()
+    device = torch.device("cuda", 0)
+    torch.cuda.set_device(0)
+    peaks, peak_kind = load_peaks()
+    Hq, Hkv, B = 28, 4, 1
+    for T, f in synth.RECTIFY_SWEEP:
+        ncache = max(1, math.ceil(300e6 / (B * Hkv * T * 512)))
+        caches = []
+        for i in range(ncache):
+            maxb = (T + BLOCK - 1) // BLOCK + 1
+            pt = synth.page_table(synth.rng(synth.RECTIFY_SWEEP_SEED + i), B, maxb)
+            cch = resa.PagedKVCache(B, Hq, Hkv, maxb, pt, device=device, zero_pools=False)
+            tg = torch.Generator(device=device)
+            tg.manual_seed(synth.RECTIFY_SWEEP_SEED * 10 + i)
+            for pool in (cch.k_pool, cch.v_pool):
+                pool.copy_(torch.randn(pool.shape, generator=tg, device=device))
+            cch.seq_lens.fill_(T)
+            resa.resa_update_summaries(cch.struct, 0, -1)
+            qn = torch.randn((B, f, Hq, HEAD_DIM), generator=tg, device=device).to(torch.bfloat16)
+            kn = torch.randn((B, f, Hkv, HEAD_DIM), generator=tg, device=device).to(torch.bfloat16)
+            vn = torch.randn((B, f, Hkv, HEAD_DIM), generator=tg, device=device).to(torch.bfloat16)
+            out = torch.empty_like(qn)
+            nb = resa.resa_workspace_size(cch.struct, 8, 0, f)
+            ws = torch.empty(nb, dtype=torch.uint8, device=device)
+            caches.append((cch, qn, kn, vn, out, ws, nb))
+        p = resa.params(0.1, 0, 0)
+
+        def one(c):
+            cch, qn, kn, vn, out, ws, nb = c
+            resa.resa_rectify_attention(cch.struct, qn, kn, vn, f, p, out, None, ws, nb)
+            resa.resa_commit_kv(cch.struct, kn, vn, f, True)
+
+        def rect_only(c):
+            cch, qn, kn, vn, out, ws, nb = c
+            resa.resa_rectify_attention(cch.struct, qn, kn, vn, f, p, out, None, ws, nb)
+        for c in caches:
+            one(c)
+        torch.cuda.synchronize()
+        reps = max(2, math.ceil(8 / ncache))
+        g_all = capture(lambda: [one(c) for _ in range(reps) for c in caches], device)
+        g_rect = capture(lambda: [rect_only(c) for _ in range(reps) for c in caches], device)
+        g_all.replay()
+        g_rect.replay()
+        calls = reps * ncache
+        t_all = time_graph(g_all, 3) / calls
+        t_rect = time_graph(g_rect, 3) / calls
+        for c in caches:
+            code, _ = resa.resa_read_device_error(c[0].struct)
+            if code:
+                raise RuntimeError(f"device error {resa.DEVICE_ERRORS.get(code)}")
+        flops = rectify_flops(B, Hq, T, f)
+        byts = rectify_bytes(B, Hq, Hkv, T, f)
+        tf = flops / t_rect / 1e12
+        gbs = byts / t_rect / 1e9
+        line = {"mode": "rectify_sweep", "context": T, "f": f, "batch": B, "caches_rotated": ncache,
+                "rectify_us": round(t_rect * 1e6, 2), "rectify_plus_overwrite_us": round(t_all * 1e6, 2),
+                "TFLOP/s": round(tf, 1), "frac_bf16_burst": round(tf / float(peaks["bf16_tflops"]), 3),
+                "frac_bf16_sustained": round(tf / float(peaks["bf16_tflops_sustained"]), 3),
+                "GB/s": round(gbs, 1), "frac_hbm": round(gbs / float(peaks["hbm_gbs"]), 3),
+                "bound": "hbm" if 7 * f < float(peaks["bf16_tflops"]) / float(peaks["hbm_gbs"]) * 1e3 else "tensor",
+                "peak_kind": peak_kind}
+        print(json.dumps(line), flush=True)
+        del caches, g_all, g_rect
+        torch.cuda.empty_cache()
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -624,6 +703,8 @@ def main():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
     ap.add_argument("--layers", type=int, default=4, help="independent layer caches rotated per decode step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--rectify-sweep", action="store_true",
+                    help="time rectification over the 16K/64K/256K x f 16/32/64 grid instead")
     ap.add_argument("--oracle-worker", default=None, help=argparse.SUPPRESS)
     ap.add_argument("--repeats", type=int, default=1, help=argparse.SUPPRESS)
     args = ap.parse_args()
@@ -634,6 +715,9 @@ def main():
     if args.warmup < 3 and args.impl == "ours":
         ap.error("--warmup must be >= 3")
     w = synth.WORKLOADS[args.workload]
+    if args.rectify_sweep:
+        run_rectify_sweep(args)
+        return
     if args.impl == "reference":
         run_reference(args, w)
     else:
