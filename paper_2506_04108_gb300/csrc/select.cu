@@ -1,20 +1,23 @@
 // Block selection (Section 2.1 "Block Selection"; Eq. 4 and Eq. 5).
 //
-// score_kernel  persistent, one CTA per SM: streams the block summaries in
-//               32 KB chunks with bulk copies through a shared-memory ring and
-//               scores them with the pooled query of the chunk's GQA group
-//               (mean of the g heads, fp32); a half-warp takes one block, a
-//               lane one 16-byte piece (8 dims) of k_min and k_max, and the
-//               128-dim sum is a fixed-order butterfly over the 16 lanes.
+// score_kernel  persistent, one CTA per SM: each of its 16 warps streams 4 KB
+//               pieces of the block summaries with its own bulk copies through
+//               its own shared-memory ring and scores them with the pooled
+//               query of the piece's GQA group (mean of the g heads, fp32); a
+//               half-warp takes one block, a lane one 16-byte piece (8 dims)
+//               of k_min and k_max, and the 128-dim sum is a fixed-order
+//               butterfly over the 16 lanes.
 // topn_kernel   one 8-CTA cluster per (sequence, KV head). The n of Eq. 5 is
 //               evaluated on the device from the device-resident length. The
-//               n-th largest order-preserving key is found by an 8-bit radix
-//               select over keys staged in the CTAs' shared memory, with the
-//               histograms summed across the cluster through distributed
-//               shared memory; the selected ids are written in ascending order
-//               by a ballot compaction that resolves ties at the threshold
-//               toward the lower block index. The last n_local blocks carry
-//               the maximum key (score +inf).
+//               last n_local blocks are always taken (score +inf); the rest
+//               of the budget is the largest order-preserving keys of the
+//               other blocks, found by a radix select over key - min key with
+//               8-bit digits from the top significant bit of the unit's key
+//               range (keys staged in the CTAs' shared memory, histograms
+//               summed across the cluster through distributed shared memory).
+//               The selected ids are written in ascending order by a ballot
+//               compaction that resolves ties at the threshold toward the
+//               lower block index.
 #include <cooperative_groups.h>
 
 #include <atomic>
@@ -25,53 +28,65 @@
 namespace resa {
 namespace {
 
-constexpr int kScoreWarps = 8;
 constexpr int kTopnCluster = 8;                                   // CTAs per (sequence, KV head)
 constexpr int kTopnThreads = 256;
 constexpr int kTopnWarps = kTopnThreads / 32;
 constexpr int kTopnSmemMax = 200 * 1024;                           // staged keys per CTA, bytes
 
-__device__ __forceinline__ float quest_term8(const float* q, const uint4& mn, const uint4& mx) {
+// Exact max of two packed bf16 pairs.
+__device__ __forceinline__ uint32_t bf16x2_max(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
+
+// Eq. 4 partial sum over 8 dims. Per dimension max(q k_max, q k_min) equals
+// |q| max(s k_max, s k_min) with s = sign(q) (scaling by |q| >= 0 and the fp32
+// rounding are monotone, so the max is taken exactly); the sign is applied to
+// the bf16 bits (`sg`), the max of two bf16 values is exact, and one fp32 FMA
+// per dimension accumulates |q| times it.
+__device__ __forceinline__ float quest_term8(const float* qa, const uint32_t* sg, const uint4& mn, const uint4& mx) {
   const uint32_t a[4] = {mn.x, mn.y, mn.z, mn.w};
   const uint32_t c[4] = {mx.x, mx.y, mx.z, mx.w};
   float s = 0.f;
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    s += fmaxf(q[2 * i] * bf16_lo(c[i]), q[2 * i] * bf16_lo(a[i]));
-    s += fmaxf(q[2 * i + 1] * bf16_hi(c[i]), q[2 * i + 1] * bf16_hi(a[i]));
+    const uint32_t m = bf16x2_max(a[i] ^ sg[i], c[i] ^ sg[i]);
+    s = fmaf(qa[2 * i], bf16_lo(m), s);
+    s = fmaf(qa[2 * i + 1], bf16_hi(m), s);
   }
   return s;
 }
 
 // Persistent score kernel: one CTA per SM. The (sequence, KV head) units'
-// summaries are cut into chunks of 64 blocks (32 KB, contiguous); CTA x owns
-// the chunk range [x * per, (x + 1) * per) of the flattened chunk list.
-// Thread 0 streams the chunks with 1-D bulk copies into a kScoreStages-deep
-// shared-memory ring; the 8 warps score each chunk from shared memory (a
-// half-warp per block, a lane per 16-byte piece of k_min and k_max, fixed
-// order 16-lane reduction) and release the stage.
-constexpr int kScoreStages = 6;
+// summaries are cut into pieces of 8 blocks (4 KB, contiguous); CTA x owns
+// the piece range [x * per, (x + 1) * per) of the flattened piece list and
+// its warp w takes every 16th piece of it (w, w + 16, ...). Each warp streams
+// its pieces with 1-D bulk copies issued by its own lane 0 through its own
+// 3-stage shared-memory ring: copies issued by one thread complete one after
+// another, so sixteen independent issuers keep enough bytes in flight per SM.
+// A half-warp scores one block, a lane one 16-byte piece (8 dims) of k_min
+// and k_max, and the 128-dim sum ends in a fixed-order 16-lane butterfly.
+constexpr int kScoreWarps = 16;
+constexpr int kScoreStages = 3;                                    // pieces in flight per warp
 constexpr int kMaxBatch = 1024;  // sequences per call supported by the score kernel
-constexpr int kChunkBlocks = 64;
-constexpr int kChunkBytes = kChunkBlocks * 2 * kHeadDim * 2;  // 32 KB
-constexpr int kScoreSmem = kScoreStages * kChunkBytes + 1024 + 2 * kScoreStages * 8 + 64;
+constexpr int kPieceBlocks = 8;
+constexpr int kPieceBytes = kPieceBlocks * 2 * kHeadDim * 2;       // 4 KB
+constexpr int kScoreRing = kScoreWarps * kScoreStages * kPieceBytes;  // 192 KB
+constexpr int kScoreSmem = kScoreRing + kScoreWarps * kScoreStages * 8;
 
-__global__ void __launch_bounds__(256, 1) score_kernel(CacheView c, const uint16_t* __restrict__ q,
-                                                       float* __restrict__ scores) {
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const uint32_t sbase = smem_u32(smem);
-  const uint32_t full0 = sbase + kScoreStages * kChunkBytes;
-  const uint32_t empty0 = full0 + 8 * kScoreStages;
-  // per-sequence block counts and the chunk prefix over (sequence, head) units
+__global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c, const uint16_t* __restrict__ q,
+                                                                    float* __restrict__ scores) {
+  extern __shared__ __align__(1024) uint8_t smem[];
+  // per-sequence block counts and the piece prefix over (sequence, head) units
   __shared__ int sh_M[kMaxBatch];
   __shared__ int sh_pref[kMaxBatch + 1];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  if (tid == 0) {
-    for (int i = 0; i < kScoreStages; ++i) {
-      mbar_init(full0 + 8 * i, 1);
-      mbar_init(empty0 + 8 * i, kScoreWarps);
-    }
+  uint8_t* ring = smem + warp * kScoreStages * kPieceBytes;
+  const uint32_t ring_s = smem_u32(ring);
+  const uint32_t bar0 = smem_u32(smem) + kScoreRing + warp * kScoreStages * 8;
+  if (lane == 0) {
+    for (int i = 0; i < kScoreStages; ++i) mbar_init(bar0 + 8 * i, 1);
     fence_mbar_init();
   }
   pdl_launch_dependents();
@@ -81,11 +96,11 @@ __global__ void __launch_bounds__(256, 1) score_kernel(CacheView c, const uint16
     sh_M[b] = (T < 0 || T > c.max_blocks * kBlock) ? 0 : (T + kBlock - 1) / kBlock;  // bad lengths: top-n reports
   }
   __syncthreads();
-  if (warp == 0) {  // exclusive prefix of Hkv * chunks-per-head over sequences
+  if (warp == 0) {  // exclusive prefix of Hkv * pieces-per-head over sequences
     int carry = 0;
     for (int b0 = 0; b0 < c.B; b0 += 32) {
       const int b = b0 + lane;
-      const int v = b < c.B ? c.Hkv * ((sh_M[b] + kChunkBlocks - 1) / kChunkBlocks) : 0;
+      const int v = b < c.B ? c.Hkv * ((sh_M[b] + kPieceBlocks - 1) / kPieceBlocks) : 0;
       int x = v;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
@@ -101,46 +116,50 @@ __global__ void __launch_bounds__(256, 1) score_kernel(CacheView c, const uint16
   const int total = sh_pref[c.B];
   const int per = (total + gridDim.x - 1) / gridDim.x;
   const int c0 = blockIdx.x * per, c1 = min(total, c0 + per);
-  const int nmine = max(0, c1 - c0);
+  const int ncta = max(0, c1 - c0);
+  const int nmine = ncta > warp ? (ncta - warp + kScoreWarps - 1) / kScoreWarps : 0;
 
-  // chunk index -> (sequence, head, first block, blocks): binary search of the prefix
-  auto locate = [&](int ci, int& b, int& h, int& blk0, int& nblk) {
+  // piece index -> (sequence, head, first block, blocks): binary search of the prefix
+  auto locate = [&](int pi, int& b, int& h, int& blk0, int& nblk) {
     int lo = 0, hi = c.B - 1;
     while (lo < hi) {
       const int mid = (lo + hi + 1) >> 1;
-      if (sh_pref[mid] <= ci) lo = mid;
+      if (sh_pref[mid] <= pi) lo = mid;
       else hi = mid - 1;
     }
     b = lo;
     const int M = sh_M[b];
-    const int per_head = (M + kChunkBlocks - 1) / kChunkBlocks;
-    const int r = ci - sh_pref[b];
+    const int per_head = (M + kPieceBlocks - 1) / kPieceBlocks;
+    const int r = pi - sh_pref[b];
     h = r / per_head;
-    blk0 = (r % per_head) * kChunkBlocks;
-    nblk = min(kChunkBlocks, M - blk0);
+    blk0 = (r % per_head) * kPieceBlocks;
+    nblk = min(kPieceBlocks, M - blk0);
   };
-  auto issue = [&](int k) {  // thread 0: my k-th chunk into stage k % kScoreStages
+  auto issue = [&](int k) {  // lane 0: this warp's k-th piece into stage k % kScoreStages
     int b, h, blk0, nblk;
-    locate(c0 + k, b, h, blk0, nblk);
-    const uint32_t bar = full0 + 8 * (k % kScoreStages);
+    locate(c0 + warp + k * kScoreWarps, b, h, blk0, nblk);
+    const uint32_t bar = bar0 + 8 * (k % kScoreStages);
     const uint32_t bytes = static_cast<uint32_t>(nblk) * 2 * kHeadDim * 2;
     mbar_arrive_expect_tx(bar, bytes);
-    bulk_load(sbase + (k % kScoreStages) * kChunkBytes,
+    bulk_load(ring_s + (k % kScoreStages) * kPieceBytes,
               c.summ + ((static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks + blk0) * 2 * kHeadDim, bytes, bar);
   };
-  if (tid == 0)
+  __syncwarp();  // lane 0's barrier initialisation precedes every lane's use
+  if (lane == 0)
     for (int k = 0; k < min(kScoreStages, nmine); ++k) issue(k);
 
   const int ch = lane & 15, half = lane >> 4;
-  int cur_unit = -1;
-  float qp[8];
+  int cur_unit = -1, k_fail = -1;
+  float qa[8];
+  uint32_t sg[4];
   for (int k = 0; k < nmine; ++k) {
     const int st = k % kScoreStages;
     int b, h, blk0, nblk;
-    locate(c0 + k, b, h, blk0, nblk);
+    locate(c0 + warp + k * kScoreWarps, b, h, blk0, nblk);
     const int unit = b * c.Hkv + h;
     if (unit != cur_unit) {  // pooled query (mean of the group's heads), this lane's 8 dims
       cur_unit = unit;
+      float qp[8];
 #pragma unroll
       for (int j = 0; j < 8; ++j) qp[j] = 0.f;
       const uint16_t* qg = q + (static_cast<size_t>(b) * c.Hq + h * c.g) * kHeadDim + ch * 8;
@@ -159,26 +178,32 @@ __global__ void __launch_bounds__(256, 1) score_kernel(CacheView c, const uint16
       }
       const float inv_g = 1.0f / static_cast<float>(c.g);
 #pragma unroll
-      for (int j = 0; j < 8; ++j) qp[j] = qp[j] * inv_g;
+      for (int j = 0; j < 4; ++j) {
+        const float lo = qp[2 * j] * inv_g, hi = qp[2 * j + 1] * inv_g;
+        qa[2 * j] = fabsf(lo);
+        qa[2 * j + 1] = fabsf(hi);
+        sg[j] = ((__float_as_uint(lo) >> 16) & 0x8000u) | (__float_as_uint(hi) & 0x80000000u);
+      }
     }
     int ok = 1;
-    if (lane == 0) ok = mbar_wait_bounded(full0 + 8 * st, (k / kScoreStages) & 1) ? 1 : 0;
+    if (lane == 0) ok = mbar_wait_bounded(bar0 + 8 * st, (k / kScoreStages) & 1) ? 1 : 0;
     ok = __shfl_sync(0xffffffffu, ok, 0);
     if (!ok) {
       if (lane == 0) record_error(c.status, RESA_DEV_WAIT_TIMEOUT, unit);
+      k_fail = k;
       break;
     }
-    mbar_try_wait(full0 + 8 * st, (k / kScoreStages) & 1);
-    const uint8_t* chunk = smem + st * kChunkBytes;
+    mbar_try_wait(bar0 + 8 * st, (k / kScoreStages) & 1);
+    const uint8_t* piece = ring + st * kPieceBytes;
     float* out = scores + static_cast<size_t>(unit) * c.max_blocks + blk0;
 #pragma unroll
-    for (int u = 0; u < kChunkBlocks / (2 * kScoreWarps); ++u) {
-      const int blk = warp * (kChunkBlocks / kScoreWarps) + 2 * u + half;
+    for (int v = 0; v < kPieceBlocks / 2; ++v) {
+      const int blk = 2 * v + half;
       float sc = 0.f;
       if (blk < nblk) {
-        const uint4 mn = *reinterpret_cast<const uint4*>(chunk + blk * 512 + ch * 16);
-        const uint4 mx = *reinterpret_cast<const uint4*>(chunk + blk * 512 + 256 + ch * 16);
-        sc = quest_term8(qp, mn, mx);
+        const uint4 mn = *reinterpret_cast<const uint4*>(piece + blk * 512 + ch * 16);
+        const uint4 mx = *reinterpret_cast<const uint4*>(piece + blk * 512 + 256 + ch * 16);
+        sc = quest_term8(qa, sg, mn, mx);
       }
       sc += __shfl_xor_sync(0xffffffffu, sc, 8);
       sc += __shfl_xor_sync(0xffffffffu, sc, 4);
@@ -186,17 +211,17 @@ __global__ void __launch_bounds__(256, 1) score_kernel(CacheView c, const uint16
       sc += __shfl_xor_sync(0xffffffffu, sc, 1);
       if (ch == 0 && blk < nblk) out[blk] = sc;
     }
-    __syncwarp();
-    if (lane == 0) mbar_arrive(empty0 + 8 * st);
-    if (tid == 0 && k + kScoreStages < nmine) {
-      // every warp has released this stage before it is refilled
-      if (!mbar_wait_bounded(empty0 + 8 * st, (k / kScoreStages) & 1)) {
-        record_error(c.status, RESA_DEV_WAIT_TIMEOUT, unit);
-      } else {
-        fence_proxy_async_smem();
-        issue(k + kScoreStages);
-      }
+    __syncwarp();  // every lane has read the stage before it is refilled
+    if (lane == 0 && k + kScoreStages < nmine) {
+      fence_proxy_async_smem();
+      issue(k + kScoreStages);
     }
+  }
+  // A warp that gave up may have copies in flight (pieces k_fail .. k_fail + 2):
+  // wait for them (bounded) before the CTA exits.
+  if (k_fail >= 0 && lane == 0) {
+    for (int k2 = k_fail; k2 < min(k_fail + kScoreStages, nmine); ++k2)
+      (void)mbar_wait_bounded(bar0 + 8 * (k2 % kScoreStages), (k2 / kScoreStages) & 1);
   }
 }
 
@@ -241,6 +266,7 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
   __shared__ int warp_a[kTopnWarps], warp_b[kTopnWarps];
   __shared__ int sh_digit, sh_rem, sh_done, sh_eq_before, sh_sel_before;
   __shared__ int cta_counts[2];  // keys above / at the boundary in this CTA, read by peers
+  __shared__ uint32_t cta_mm[2];  // this CTA's smallest and largest unforced key, read by peers
   namespace cg = cooperative_groups;
   cg::cluster_group cluster = cg::this_cluster();
   pdl_launch_dependents();
@@ -272,7 +298,11 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
   const int per = (M + kTopnCluster - 1) / kTopnCluster;
   const int lo = rank * per, cnt = max(0, min(M, lo + per) - lo);
   const float* sc = scores + (static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks + lo;
-  const int first_forced = M - n_local - lo;
+  const int F = M - min(n_local, M);  // blocks [F, M) are forced (score +inf)
+  const int nf = min(M - F, n);       // forced blocks taken (all unless n was clamped)
+  const int r = n - nf;               // blocks to pick among [0, F)
+  const int f_loc = F - lo;           // this CTA's ids >= f_loc are forced
+  uint32_t kmin = 0xFFFFFFFFu, kmax = 0u;
   for (int i0 = 0; i0 < cnt; i0 += 4 * kTopnThreads) {  // four loads in flight per thread
     float v[4];
 #pragma unroll
@@ -283,26 +313,64 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       const int i = i0 + u * kTopnThreads + tid;
-      if (i < cnt) keys[i] = (i >= first_forced) ? 0xFFFFFFFFu : score_key(v[u]);
+      if (i < cnt) {
+        const uint32_t k = score_key(v[u]);
+        keys[i] = k;
+        if (i < f_loc) {
+          kmin = min(kmin, k);
+          kmax = max(kmax, k);
+        }
+      }
     }
   }
   const int cnt_round = (cnt + 31) / 32 * 32;
-
-  // ---- radix select of the n-th largest key across the cluster ----
-  uint32_t prefix = 0, pmask = 0;
-  int rem = n;
+  // extreme unforced keys of the unit: CTA reduction, then across the cluster
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    kmin = min(kmin, __shfl_xor_sync(0xffffffffu, kmin, o));
+    kmax = max(kmax, __shfl_xor_sync(0xffffffffu, kmax, o));
+  }
+  if (lane == 0) {
+    warp_a[warp] = static_cast<int>(kmin);
+    warp_b[warp] = static_cast<int>(kmax);
+  }
   __syncthreads();
-  if (n > 0) {
-    for (int pass = 0; pass < 4; ++pass) {
-      const int shift = 24 - 8 * pass;
+  if (tid == 0) {
+    uint32_t a = 0xFFFFFFFFu, z = 0u;
+    for (int w = 0; w < kTopnWarps; ++w) {
+      a = min(a, static_cast<uint32_t>(warp_a[w]));
+      z = max(z, static_cast<uint32_t>(warp_b[w]));
+    }
+    cta_mm[0] = a;
+    cta_mm[1] = z;
+  }
+  cluster.sync();  // every CTA's extremes are visible
+#pragma unroll
+  for (int q = 0; q < kTopnCluster; ++q) {
+    const uint32_t* pm = cluster.map_shared_rank(cta_mm, q);
+    kmin = min(kmin, pm[0]);
+    kmax = max(kmax, pm[1]);
+  }
+
+  // ---- radix select of the r-th largest v = key - kmin among blocks [0, F) ----
+  // The first digit is the top 8 significant bits of v, so the digits adapt
+  // to the range of the unit's scores (which sit within a few per cent of
+  // each other); r == 0 or r == F need no pass (prefix = pmask = 0).
+  uint32_t prefix = 0, pmask = 0;
+  int rem = r;
+  if (r > 0 && r < F) {
+    const int bits = 32 - __clz(static_cast<int>(kmax - kmin));  // significant bits of v
+    int shift = max(bits - 8, 0), width = bits - shift;
+    for (int pass = 0;; ++pass) {
+      const uint32_t dmask = (1u << width) - 1u;
       int* hb = hist[pass & 1];
       hb[tid] = 0;
       __syncthreads();
       for (int i = tid; i < cnt_round; i += kTopnThreads) {
         uint32_t d = 0x100u;  // sentinel: not counted
-        if (i < cnt) {
-          const uint32_t k = keys[i];
-          if ((k & pmask) == prefix) d = (k >> shift) & 0xFFu;
+        if (i < cnt && i < f_loc) {
+          const uint32_t v = keys[i] - kmin;
+          if ((v & pmask) == prefix) d = (v >> shift) & dmask;
         }
         const unsigned peers = __match_any_sync(0xffffffffu, d);
         if (d != 0x100u && lane == __ffs(peers) - 1) atomicAdd(&hb[d], __popc(peers));
@@ -344,14 +412,30 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
       }
       __syncthreads();
       prefix |= static_cast<uint32_t>(sh_digit) << shift;
-      pmask |= 0xFFu << shift;
+      pmask |= dmask << shift;
       rem = sh_rem;
-      if (sh_done) break;  // identical decision in every CTA of the cluster
+      if (sh_done || shift == 0) break;  // identical decision in every CTA of the cluster
+      width = min(8, shift);
+      shift -= width;
     }
   }
-  // Selected: (key & pmask) > prefix, or == prefix among the first `take_eq`
-  // such keys in block order.
-  const int take_eq = n > 0 ? rem : 0;
+  // Selected: forced blocks [F, F + nf), and among [0, F) the ids with
+  // (v & pmask) > prefix, or == prefix among the first `take_eq` such ids in
+  // block order.
+  const int take_eq = rem;
+  auto classify = [&](int i, bool in, bool& is_gt, bool& is_eq) {  // local id i
+    is_gt = false;
+    is_eq = false;
+    if (in) {
+      if (i >= f_loc) {
+        is_gt = lo + i - F < nf;
+      } else {
+        const uint32_t v = (keys[i] - kmin) & pmask;
+        is_gt = v > prefix;
+        is_eq = v == prefix;
+      }
+    }
+  };
 
   // ---- ordered compaction: warps own contiguous id ranges of the CTA ----
   const int per_warp = (cnt_round / 32 + kTopnWarps - 1) / kTopnWarps * 32;
@@ -360,10 +444,10 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
   if (n > 0) {
     for (int i0 = w0; i0 < w0 + per_warp; i0 += 32) {
       const int i = i0 + lane;
-      const bool in = i < w1;
-      const uint32_t k = in ? (keys[i] & pmask) : 0u;
-      gt += __popc(__ballot_sync(0xffffffffu, in && k > prefix));
-      eq += __popc(__ballot_sync(0xffffffffu, in && k == prefix));
+      bool is_gt, is_eq;
+      classify(i, i < w1, is_gt, is_eq);
+      gt += __popc(__ballot_sync(0xffffffffu, is_gt));
+      eq += __popc(__ballot_sync(0xffffffffu, is_eq));
     }
   }
   if (lane == 0) {
@@ -407,12 +491,11 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
     int pos = sh_sel_before + warp_b[warp];
     for (int i0 = w0; i0 < w0 + per_warp; i0 += 32) {
       const int i = i0 + lane;
-      const bool in = i < w1;
-      const uint32_t k = in ? (keys[i] & pmask) : 0u;
-      const bool is_eq = in && k == prefix;
+      bool is_gt, is_eq;
+      classify(i, i < w1, is_gt, is_eq);
       const unsigned eqm = __ballot_sync(0xffffffffu, is_eq);
       const int my_eq_rank = eq_seen + __popc(eqm & ((1u << lane) - 1u));
-      const bool sel = in && (k > prefix || (is_eq && my_eq_rank < take_eq));
+      const bool sel = is_gt || (is_eq && my_eq_rank < take_eq);
       const unsigned selm = __ballot_sync(0xffffffffu, sel);
       if (sel) out[pos + __popc(selm & ((1u << lane) - 1u))] = lo + i;
       eq_seen += __popc(eqm);
@@ -437,9 +520,10 @@ cudaError_t launch_select(const CacheView& c, const uint16_t* q, double keep, in
                           cudaStream_t st) {
   cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(score_kernel), kScoreSmem, 3);
   if (e != cudaSuccess) return e;
-  // one persistent CTA per SM (never more than the chunks there can be)
-  const int max_chunks = c.B * c.Hkv * ((c.max_blocks + kChunkBlocks - 1) / kChunkBlocks);
-  const int grid = max(1, min(sm_count, max_chunks));
+  // one persistent CTA per SM (never more than the pieces there can be)
+  const long long max_pieces =
+      static_cast<long long>(c.B) * c.Hkv * ((c.max_blocks + kPieceBlocks - 1) / kPieceBlocks);
+  const int grid = static_cast<int>(max(1LL, min(static_cast<long long>(sm_count), max_pieces)));
   e = launch_pdl(score_kernel, dim3(grid), dim3(kScoreWarps * 32), kScoreSmem, st, c, q, scores);
   if (e != cudaSuccess) return e;
   const size_t smem = select_smem_bytes(c.max_blocks);

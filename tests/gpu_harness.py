@@ -86,6 +86,8 @@ def check_selection(gpu_sel, scores, n, n_local):
     M = len(scores)
     assert len(gpu_sel) == n, (len(gpu_sel), n)
     assert len(set(gpu_sel.tolist())) == n
+    if n == 0:
+        return True
     assert np.all(np.diff(gpu_sel) > 0), "indices must be ascending"
     assert gpu_sel.min() >= 0 and gpu_sel.max() < M
     want = O.select_blocks(scores, n, n_local)

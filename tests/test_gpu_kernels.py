@@ -133,6 +133,54 @@ def test_select_matches_oracle(g, Hkv, lens, keep, n_min, n_local):
             H.check_selection(idx[b, h, :n], scores, n, n_local)
 
 
+def check_select_case(cache, Ks, Vs, q, p, maxb, idx, cnt):
+    g = cache.Hq // cache.Hkv
+    for b, Kb in enumerate(Ks):
+        st = H.oracle_state(Kb, Vs[b], maxb * 16)
+        for h in range(cache.Hkv):
+            sel, scores, n = O.select_for_group(st, h, O.widen_bf16(q[b, h * g:(h + 1) * g]),
+                                                O.ResaParams(p.keep_ratio, p.n_min_blocks, p.n_local_blocks))
+            assert cnt[b, h] == n
+            assert np.all(idx[b, h, n:] == -1)
+            H.check_selection(idx[b, h, :n], scores, n, p.n_local_blocks)
+
+
+def test_select_many_small_units_and_repeat():
+    """More (sequence, KV head) units than SMs, of one or two score pieces
+    each, ragged lengths and two empty sequences (count 0, ids -1). A second
+    call on the same state must give the same result."""
+    B, Hkv, g = 100, 2, 4
+    lens = [int(x) for x in synth.rng(71).integers(1, 1100, size=B)]
+    lens[3] = 0
+    lens[50] = 0
+    Ks, Vs = seq_inputs(72, B, Hkv, lens)
+    maxb = 72
+    cache = H.make_cache(Ks, Vs, g * Hkv, maxb)
+    q = synth.normal_bf16(synth.rng(73), (B, g * Hkv, 128))
+    p = resa.params(0.2, 2, 1)
+    n_cap = resa.resa_max_selected(cache.struct, p)
+    idx, cnt = run_select(cache, q, p, n_cap)
+    assert resa.resa_read_device_error(cache.struct) == (0, 0)
+    check_select_case(cache, Ks, Vs, q, p, maxb, idx, cnt)
+    idx2, cnt2 = run_select(cache, q, p, n_cap)
+    assert np.array_equal(idx, idx2) and np.array_equal(cnt, cnt2)
+
+
+def test_select_large_unit():
+    """One unit of 30,001 blocks (3,751 keys staged per CTA of the cluster)."""
+    M = 30001
+    T = M * 16 - 7
+    Ks, Vs = seq_inputs(74, 1, 1, [T])
+    maxb = M + 3
+    cache = H.make_cache(Ks, Vs, 2, maxb)
+    q = synth.normal_bf16(synth.rng(75), (1, 2, 128))
+    p = resa.params(0.05, 16, 4)
+    n_cap = resa.resa_max_selected(cache.struct, p)
+    idx, cnt = run_select(cache, q, p, n_cap)
+    assert resa.resa_read_device_error(cache.struct) == (0, 0)
+    check_select_case(cache, Ks, Vs, q, p, maxb, idx, cnt)
+
+
 def test_select_ties_go_to_lower_index():
     """Identical blocks give identical scores; the lower ids must win."""
     Hkv, g, T = 1, 4, 16 * 40
