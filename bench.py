@@ -694,6 +694,84 @@ def run_rectify_sweep(args):
         torch.cuda.empty_cache()
 
 
+def run_breakdown(args):
+    """Per-call latency breakdown of one layer-step at batch 8 (28 q / 4 KV
+    heads, d 128, keep 0.1, n_min 128 blocks, n_local 1, f 32) for each
+    context in synth.BREAKDOWN_CONTEXTS, next to dense flash decoding of the
+    same step (the sparse-decode kernel given every block of the sequence).
+    The sparse step is commit + select + sparse decode + (rectify +
+    overwrite) / f; the dense step is commit + dense decode. Enough caches
+    rotate per context that the rotation exceeds L2. One JSON line per
+    context."""
+    import dataclasses
+    import torch
+    from paper_2506_04108_gb300 import build as _b
+    from paper_2506_04108_gb300 import resa
+    _b.build()
+    resa.load()
+    device = torch.device("cuda", 0)
+    torch.cuda.set_device(0)
+    peaks, peak_kind = load_peaks()
+    hbm = float(peaks["hbm_gbs"])
+    base = synth.WORKLOADS[DEFAULT_WORKLOAD]
+    for T0 in synth.BREAKDOWN_CONTEXTS:
+        w = dataclasses.replace(base, name=f"breakdown_b8_ctx{T0 // 1024}k", context=T0)
+        B, Hq, Hkv, f = w.batch, w.num_q_heads, w.num_kv_heads, w.f
+        ncache = max(1, math.ceil(400e6 / (B * Hkv * T0 * 512)))
+        capacity = ((T0 + f * (2 + 2 * ATTR_REPS) + BLOCK) // BLOCK + 1) * BLOCK
+        layers = [LayerCache(w, capacity, w.seed * 100 + 31 * i, device) for i in range(ncache)]
+        run_period(layers)                       # warm-up, appends f tokens
+        T = T0 + f
+        torch.cuda.synchronize()
+        # dense selection: every block of every sequence, in order
+        M = (T + BLOCK - 1) // BLOCK
+        maxb = layers[0].cache.max_blocks
+        dense_idx = torch.arange(maxb, dtype=torch.int32, device=device).expand(B, Hkv, maxb).contiguous()
+        dense_cnt = torch.full((B, Hkv), M, dtype=torch.int32, device=device)
+        dense_ws = []
+        for Lc in layers:
+            nb = resa.resa_workspace_size(Lc.cache.struct, maxb, 0, 0)
+            dense_ws.append((torch.empty(nb, dtype=torch.uint8, device=device), nb))
+
+        def dense(i, t):
+            Lc = layers[i]
+            ws, nb = dense_ws[i]
+            resa.resa_sparse_decode(Lc.cache.struct, Lc.q[t], dense_idx, dense_cnt, maxb, Lc.p, Lc.out[t], None, 0,
+                                    ws, nb)
+        kinds = {
+            "select": (lambda: [Lc.select(t) for t in range(f) for Lc in layers], f),
+            "decode": (lambda: [Lc.sparse_decode(t) for t in range(f) for Lc in layers], f),
+            "dense_decode": (lambda: [dense(i, t) for t in range(f) for i in range(len(layers))], f),
+            "rectify": (lambda: [Lc.rectify_attention() for Lc in layers], 1),
+            "overwrite": (lambda: [Lc.overwrite() for Lc in layers], 1),
+            "commit": (lambda: [Lc.commit(t) for t in range(f) for Lc in layers], f),
+        }
+        us = {}
+        for kind, (fn, per_layer) in kinds.items():
+            gk = capture(fn, device)
+            gk.replay()
+            us[kind] = time_graph(gk, ATTR_REPS) / (per_layer * len(layers)) * 1e6
+            del gk
+        check_device_errors(layers)
+        sparse = us["commit"] + us["select"] + us["decode"] + (us["rectify"] + us["overwrite"]) / f
+        dense_step = us["commit"] + us["dense_decode"]
+        dense_bytes = B * Hkv * T * 512 + B * Hq * HEAD_DIM * 4
+        sparse_bytes = decode_bytes(B, Hq, Hkv, T, w.keep, w.n_min_blocks, w.n_local_blocks)
+        line = {"mode": "breakdown", "context": T0, "batch": B, "q_heads": Hq, "kv_heads": Hkv, "keep": w.keep,
+                "f": f, "caches_rotated": ncache,
+                "us_per_call": {k: round(v, 2) for k, v in us.items()},
+                "sparse_step_us": round(sparse, 2), "dense_step_us": round(dense_step, 2),
+                "dense_over_sparse": round(dense_step / sparse, 2),
+                "dense_decode_GB/s": round(dense_bytes / (us["dense_decode"] * 1e-6) / 1e9, 1),
+                "dense_decode_frac_hbm": round(dense_bytes / (us["dense_decode"] * 1e-6) / 1e9 / hbm, 3),
+                "sparse_decode_GB/s": round(sparse_bytes / (us["decode"] * 1e-6) / 1e9, 1),
+                "sparse_decode_frac_hbm": round(sparse_bytes / (us["decode"] * 1e-6) / 1e9 / hbm, 3),
+                "peak_kind": peak_kind, "data": "synthetic"}
+        print(json.dumps(line), flush=True)
+        del layers, dense_ws, dense_idx
+        torch.cuda.empty_cache()
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -703,6 +781,8 @@ def main():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
     ap.add_argument("--layers", type=int, default=4, help="independent layer caches rotated per decode step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--breakdown", action="store_true",
+                    help="per-call latency breakdown versus dense decoding at 16K/64K/256K, batch 8")
     ap.add_argument("--rectify-sweep", action="store_true",
                     help="time rectification over the 16K/64K/256K x f 16/32/64 grid instead")
     ap.add_argument("--oracle-worker", default=None, help=argparse.SUPPRESS)
@@ -717,6 +797,9 @@ def main():
     w = synth.WORKLOADS[args.workload]
     if args.rectify_sweep:
         run_rectify_sweep(args)
+        return
+    if args.breakdown:
+        run_breakdown(args)
         return
     if args.impl == "reference":
         run_reference(args, w)

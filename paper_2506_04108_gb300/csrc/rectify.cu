@@ -14,8 +14,9 @@
 //
 // CTA = 12 warps:
 //   warp 0      TMA producer: 64-key K and V tiles of the prefix, one
-//               SWIZZLE_128B box per 16-key page per 64-column half, into a
-//               5-stage ring (kv_full / kv_empty mbarriers); the causal tail
+//               SWIZZLE_128B box per 16-key page per 64-column half, issued
+//               by 16 lanes, into a 5-stage ring (kv_full / kv_empty
+//               mbarriers); page ids are read 32 blocks at a time; the causal tail
 //               is written by the warp's lanes in the same swizzled layout.
 //   warp 1      allocates 512 TMEM columns; lane 0 issues the MMAs:
 //               S[t] = Q K^T (M 128, N 64, K 128; both operands K-major from
@@ -171,6 +172,9 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
 
   if (warp == 0) {
     // ------------------------------------------------------- producer ---
+    // Page rows of the prefix blocks are read 32 at a time (8 tiles, one
+    // block per lane) and the 16 boxes of a tile are issued by 16 lanes.
+    int win = -1, my_row = -1;
     for (int t = 0; t < n_tiles; ++t) {
       const int st = t % kStages;
       if (t >= kStages && !warp_wait(bar(kBarKvEmpty + st), ((t / kStages) - 1) & 1)) {
@@ -180,30 +184,29 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
       uint8_t* kst = smem + kOffKV + st * kStageBytes;
       const uint32_t kdst = sbase + kOffKV + st * kStageBytes;
       if (t < n_pref) {
-        if (lane == 0) {
-          const int kb = (t0 + t) * kTileKeys;
-          int rows[4], pages = 0;
-          for (int pg = 0; pg < 4; ++pg) {
-            rows[pg] = -1;
-            const int blk = kb / kBlock + pg;
-            if (blk * kBlock >= P) continue;
+        if ((t & ~7) != win) {
+          win = t & ~7;
+          const int blk = (t0 + win) * (kTileKeys / kBlock) + lane;
+          my_row = -1;
+          if (blk * kBlock < P) {
             const int page = c.page_table[static_cast<size_t>(b) * c.max_blocks + blk];
-            if (page < 0 || page >= c.num_pages) {
-              record_error(c.status, RESA_DEV_PAGE_RANGE, b);
-              continue;
-            }
-            rows[pg] = (page * c.Hkv + h) * kBlock;
-            ++pages;
+            if (page >= 0 && page < c.num_pages)
+              my_row = (page * c.Hkv + h) * kBlock;
+            else if (win * (kTileKeys / kBlock) + lane < n_pref * (kTileKeys / kBlock))
+              record_error(c.status, RESA_DEV_PAGE_RANGE, b);  // a block this CTA uses: left out
           }
-          mbar_arrive_expect_tx(bar(kBarKvFull + st), pages * 4 * 2048);
-          for (int pg = 0; pg < 4; ++pg) {
-            if (rows[pg] < 0) continue;
-            const uint32_t o = pg * 2048;
-            tma_load_2d(kdst + o, &tm_k, bar(kBarKvFull + st), 0, rows[pg]);
-            tma_load_2d(kdst + kKVHalf + o, &tm_k, bar(kBarKvFull + st), 64, rows[pg]);
-            tma_load_2d(kdst + 2 * kKVHalf + o, &tm_v, bar(kBarKvFull + st), 0, rows[pg]);
-            tma_load_2d(kdst + 3 * kKVHalf + o, &tm_v, bar(kBarKvFull + st), 64, rows[pg]);
-          }
+        }
+        const int slot = (t - win) * (kTileKeys / kBlock);
+        int pages = 0;
+#pragma unroll
+        for (int pg = 0; pg < kTileKeys / kBlock; ++pg) pages += __shfl_sync(0xffffffffu, my_row, slot + pg) >= 0 ? 1 : 0;
+        const int row = __shfl_sync(0xffffffffu, my_row, slot + ((lane >> 2) & 3));
+        if (lane == 0) mbar_arrive_expect_tx(bar(kBarKvFull + st), pages * 4 * 2048);
+        __syncwarp();
+        if (lane < 16 && row >= 0) {  // lane 4 pg + part: part 0/1 = K halves, 2/3 = V halves
+          const int part = lane & 3;
+          tma_load_2d(kdst + part * kKVHalf + (lane >> 2) * 2048, part < 2 ? &tm_k : &tm_v, bar(kBarKvFull + st),
+                      (part & 1) * 64, row);
         }
       } else {
         const int tb = (t - n_pref) * kTileKeys;  // tail tile: tokens tb .. tb + 63 of the f

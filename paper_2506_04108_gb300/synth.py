@@ -136,6 +136,10 @@ WORKLOADS = {
         steps=512, f=32, keep=0.05, n_min_blocks=128, n_local_blocks=1, seed=2506041084),
 }
 
+# Latency breakdown (sparse step versus dense flash decoding of every block):
+# the 32K batch-8 workload's geometry and ReSA parameters at these contexts.
+BREAKDOWN_CONTEXTS = (16384, 65536, 262144)
+
 # Rectification-only sweep: f new queries against cached contexts.
 RECTIFY_SWEEP = [(t, f) for t in (16384, 65536, 262144) for f in (16, 32, 64)]
 RECTIFY_SWEEP_SEED = 2506041085
