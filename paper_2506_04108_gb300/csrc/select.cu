@@ -89,36 +89,32 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c,
     for (int i = 0; i < kScoreStages; ++i) mbar_init(bar0 + 8 * i, 1);
     fence_mbar_init();
   }
-  pdl_launch_dependents();
-  pdl_wait();
-  for (int b = tid; b < c.B; b += blockDim.x) {
-    const int T = c.seq_lens[b];
-    sh_M[b] = (T < 0 || T > c.max_blocks * kBlock) ? 0 : (T + kBlock - 1) / kBlock;  // bad lengths: top-n reports
-  }
-  __syncthreads();
-  if (warp == 0) {  // exclusive prefix of Hkv * pieces-per-head over sequences
-    int carry = 0;
-    for (int b0 = 0; b0 < c.B; b0 += 32) {
-      const int b = b0 + lane;
-      const int v = b < c.B ? c.Hkv * ((sh_M[b] + kPieceBlocks - 1) / kPieceBlocks) : 0;
-      int x = v;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, x, o);
-        if (lane >= o) x += y;
-      }
-      if (b < c.B) sh_pref[b] = carry + x - v;
-      carry += __shfl_sync(0xffffffffu, x, 31);
+  // per-sequence block counts and the exclusive prefix of Hkv * pieces-per-head
+  // over sequences (lengths out of range count as empty: top-n reports them)
+  auto build_tables = [&]() {
+    for (int b = tid; b < c.B; b += blockDim.x) {
+      const int T = c.seq_lens[b];
+      sh_M[b] = (T < 0 || T > c.max_blocks * kBlock) ? 0 : (T + kBlock - 1) / kBlock;
     }
-    if (lane == 0) sh_pref[c.B] = carry;
-  }
-  __syncthreads();
-  const int total = sh_pref[c.B];
-  const int per = (total + gridDim.x - 1) / gridDim.x;
-  const int c0 = blockIdx.x * per, c1 = min(total, c0 + per);
-  const int ncta = max(0, c1 - c0);
-  const int nmine = ncta > warp ? (ncta - warp + kScoreWarps - 1) / kScoreWarps : 0;
-
+    __syncthreads();
+    if (warp == 0) {
+      int carry = 0;
+      for (int b0 = 0; b0 < c.B; b0 += 32) {
+        const int b = b0 + lane;
+        const int v = b < c.B ? c.Hkv * ((sh_M[b] + kPieceBlocks - 1) / kPieceBlocks) : 0;
+        int x = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int y = __shfl_up_sync(0xffffffffu, x, o);
+          if (lane >= o) x += y;
+        }
+        if (b < c.B) sh_pref[b] = carry + x - v;
+        carry += __shfl_sync(0xffffffffu, x, 31);
+      }
+      if (lane == 0) sh_pref[c.B] = carry;
+    }
+    __syncthreads();
+  };
   // piece index -> (sequence, head, first block, blocks): binary search of the prefix
   auto locate = [&](int pi, int& b, int& h, int& blk0, int& nblk) {
     int lo = 0, hi = c.B - 1;
@@ -135,6 +131,35 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c,
     blk0 = (r % per_head) * kPieceBlocks;
     nblk = min(kPieceBlocks, M - blk0);
   };
+  pdl_launch_dependents();
+  // Before the wait for the preceding kernel, prefetch this warp's pieces into
+  // L2 from the lengths as they are now (the append commit that may still be
+  // running changes at most the last block of a sequence; a stale length only
+  // misses or adds a prefetch, and addresses stay inside the summaries).
+  build_tables();
+  {
+    const int total = sh_pref[c.B];
+    const int per = (total + gridDim.x - 1) / gridDim.x;
+    const int c0 = blockIdx.x * per, c1 = min(total, c0 + per);
+    const int ncta = max(0, c1 - c0);
+    const int nmine = ncta > warp ? (ncta - warp + kScoreWarps - 1) / kScoreWarps : 0;
+    if (lane == 0)
+      for (int k = 0; k < nmine; ++k) {
+        int b, h, blk0, nblk;
+        locate(c0 + warp + k * kScoreWarps, b, h, blk0, nblk);
+        bulk_prefetch_l2(c.summ + ((static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks + blk0) * 2 * kHeadDim,
+                         static_cast<uint32_t>(nblk) * 2 * kHeadDim * 2);
+      }
+  }
+  __syncthreads();  // the tables are rebuilt below
+  pdl_wait();
+  build_tables();
+  const int total = sh_pref[c.B];
+  const int per = (total + gridDim.x - 1) / gridDim.x;
+  const int c0 = blockIdx.x * per, c1 = min(total, c0 + per);
+  const int ncta = max(0, c1 - c0);
+  const int nmine = ncta > warp ? (ncta - warp + kScoreWarps - 1) / kScoreWarps : 0;
+
   auto issue = [&](int k) {  // lane 0: this warp's k-th piece into stage k % kScoreStages
     int b, h, blk0, nblk;
     locate(c0 + warp + k * kScoreWarps, b, h, blk0, nblk);
