@@ -772,6 +772,64 @@ def run_breakdown(args):
         torch.cuda.empty_cache()
 
 
+def run_prefill(args):
+    """Chunked dense prefill (Algorithm 1's prefill): for each chunk of the
+    prompt, the append commit of its K/V (block keys built online) and the
+    rectification call with f = chunk, which attends the chunk's queries
+    causally to the cached prefix and the chunk. Batch 1, 28 q / 4 KV heads,
+    d 128, chunks of synth.PREFILL_CHUNK tokens; the whole prompt is one CUDA
+    graph. One JSON line per prompt length (tokens/s and TFLOP/s of the useful
+    causal flops, 4 d Hq L^2 / 2 + O(L))."""
+    import torch
+    from paper_2506_04108_gb300 import build as _b
+    from paper_2506_04108_gb300 import resa
+    _b.build()
+    resa.load()
+    device = torch.device("cuda", 0)
+    torch.cuda.set_device(0)
+    peaks, peak_kind = load_peaks()
+    Hq, Hkv, B, C = 28, 4, 1, synth.PREFILL_CHUNK
+    for L in synth.PREFILL_LENGTHS:
+        maxb = (L + BLOCK - 1) // BLOCK + 1
+        pt = synth.page_table(synth.rng(synth.PREFILL_SEED), B, maxb)
+        cch = resa.PagedKVCache(B, Hq, Hkv, maxb, pt, device=device, zero_pools=False)
+        tg = torch.Generator(device=device)
+        tg.manual_seed(synth.PREFILL_SEED)
+        q = torch.randn((B, L, Hq, HEAD_DIM), generator=tg, device=device).to(torch.bfloat16)
+        k = torch.randn((B, L, Hkv, HEAD_DIM), generator=tg, device=device).to(torch.bfloat16)
+        v = torch.randn((B, L, Hkv, HEAD_DIM), generator=tg, device=device).to(torch.bfloat16)
+        out = torch.empty_like(q)
+        nb = resa.resa_workspace_size(cch.struct, 8, 0, C)
+        ws = torch.empty(nb, dtype=torch.uint8, device=device)
+        p = resa.params(0.1, 0, 0)
+        chunks = [(c0, min(C, L - c0)) for c0 in range(0, L, C)]
+        # per chunk: contiguous [B, f, H, d] views (slices of [B, L, H, d] are contiguous for B = 1)
+        views = [(q[:, c0:c0 + f], k[:, c0:c0 + f], v[:, c0:c0 + f], out[:, c0:c0 + f], f) for c0, f in chunks]
+
+        def prefill():
+            cch.seq_lens.zero_()
+            for qc, kc, vc, oc, f in views:
+                resa.resa_commit_kv(cch.struct, kc, vc, f, False)
+                resa.resa_rectify_attention(cch.struct, qc, kc, vc, f, p, oc, None, ws, nb)
+        prefill()
+        torch.cuda.synchronize()
+        g = capture(prefill, device)
+        g.replay()
+        secs = time_graph(g, 3)
+        code, _ = resa.resa_read_device_error(cch.struct)
+        if code:
+            raise RuntimeError(f"device error {resa.DEVICE_ERRORS.get(code)}")
+        flops = 4.0 * HEAD_DIM * Hq * B * (L * (L + 1) / 2)
+        tf = flops / secs / 1e12
+        print(json.dumps({"mode": "prefill", "prompt": L, "chunk": C, "batch": B, "q_heads": Hq, "kv_heads": Hkv,
+                          "ms": round(secs * 1e3, 3), "tokens/s": round(B * L / secs, 1),
+                          "TFLOP/s": round(tf, 1), "frac_bf16_burst": round(tf / float(peaks["bf16_tflops"]), 3),
+                          "frac_bf16_sustained": round(tf / float(peaks["bf16_tflops_sustained"]), 3),
+                          "peak_kind": peak_kind, "data": "synthetic"}), flush=True)
+        del cch, q, k, v, out, ws, g
+        torch.cuda.empty_cache()
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -781,6 +839,7 @@ def main():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
     ap.add_argument("--layers", type=int, default=4, help="independent layer caches rotated per decode step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--prefill", action="store_true", help="chunked dense prefill throughput (32K, 128K prompts)")
     ap.add_argument("--breakdown", action="store_true",
                     help="per-call latency breakdown versus dense decoding at 16K/64K/256K, batch 8")
     ap.add_argument("--rectify-sweep", action="store_true",
@@ -800,6 +859,9 @@ def main():
         return
     if args.breakdown:
         run_breakdown(args)
+        return
+    if args.prefill:
+        run_prefill(args)
         return
     if args.impl == "reference":
         run_reference(args, w)

@@ -233,6 +233,10 @@ resa_status_t resa_sparse_decode(const resa_cache_t* cache, const void* q, const
  *   out       bf16 [batch][f][num_q_heads][head_dim]
  *   lse       fp32 [batch][f][num_q_heads] or NULL (natural log).
  * Device errors: seq_lens[b] < f records RESA_DEV_SEQ_LEN_RANGE.
+ * The same call is the attention of Algorithm 1's dense prefill done in
+ * chunks: after resa_commit_kv(append) of a chunk of C prompt tokens (which
+ * also builds their block keys), f = C attends the chunk's queries causally
+ * to the cached prefix and to the chunk itself.
  */
 resa_status_t resa_rectify_attention(const resa_cache_t* cache, const void* q_new, const void* k_new,
                                      const void* v_new, int32_t f, const resa_params_t* params, void* out,

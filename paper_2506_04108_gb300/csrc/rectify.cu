@@ -16,8 +16,10 @@
 //   warp 0      TMA producer: 64-key K and V tiles of the prefix, one
 //               SWIZZLE_128B box per 16-key page per 64-column half, issued
 //               by 16 lanes, into a 5-stage ring (kv_full / kv_empty
-//               mbarriers); page ids are read 32 blocks at a time; the causal tail
-//               is written by the warp's lanes in the same swizzled layout.
+//               mbarriers); page ids are read 32 blocks at a time. The
+//               tiles of the f new tokens come from k_new / v_new by 4-D TMA
+//               boxes (64 tokens x 64 dims of one head), only up to the last
+//               token of the CTA's rows (later keys are causally masked).
 //   warp 1      allocates 512 TMEM columns; lane 0 issues the MMAs:
 //               S[t] = Q K^T (M 128, N 64, K 128; both operands K-major from
 //               shared memory) into a double-buffered TMEM S, and
@@ -93,6 +95,8 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity) {
 
 __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_constant__ CUtensorMap tm_k,
                                                               const __grid_constant__ CUtensorMap tm_v,
+                                                              const __grid_constant__ CUtensorMap tm_kn,
+                                                              const __grid_constant__ CUtensorMap tm_vn,
                                                               CacheView c, RectArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -123,6 +127,8 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
     fence_mbar_init();
     prefetch_tmap(&tm_k);
     prefetch_tmap(&tm_v);
+    prefetch_tmap(&tm_kn);
+    prefetch_tmap(&tm_vn);
   }
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), kTmemCols);
@@ -142,7 +148,10 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
   const int per = (ntp + a.splits - 1) / a.splits;
   const int t0 = s * per;
   const int n_pref = max(0, min(ntp, t0 + per) - t0);
-  const int n_tail = (!bad && s == a.splits - 1) ? (f + kTileKeys - 1) / kTileKeys : 0;
+  // tail tiles of the f new tokens, up to the last token of this CTA's rows
+  // (later keys are causally masked for every row here)
+  const int tok_end = min(f, (row0 + MT * kMTile + 7) / 8);
+  const int n_tail = (!bad && s == a.splits - 1) ? (tok_end + kTileKeys - 1) / kTileKeys : 0;
   const int n_tiles = n_pref + n_tail;
   if (bad && tid == 0 && s == 0 && rg == 0) record_error(c.status, RESA_DEV_SEQ_LEN_RANGE, b);
 
@@ -181,7 +190,6 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
         if (lane == 0) record_error(c.status, RESA_DEV_WAIT_TIMEOUT, bh);
         break;
       }
-      uint8_t* kst = smem + kOffKV + st * kStageBytes;
       const uint32_t kdst = sbase + kOffKV + st * kStageBytes;
       if (t < n_pref) {
         if ((t & ~7) != win) {
@@ -209,22 +217,16 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
                       (part & 1) * 64, row);
         }
       } else {
-        const int tb = (t - n_pref) * kTileKeys;  // tail tile: tokens tb .. tb + 63 of the f
-        for (int e = lane; e < kTileKeys * 16; e += 32) {
-          const int row = e >> 4, ch = e & 15, tok = tb + row;
-          uint4 kv = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
-          if (tok < f) {
-            const size_t src = ((static_cast<size_t>(b) * f + tok) * c.Hkv + h) * kHeadDim + ch * 8;
-            kv = *reinterpret_cast<const uint4*>(a.k_new + src);
-            vv = *reinterpret_cast<const uint4*>(a.v_new + src);
-          }
-          const uint32_t off = (ch >> 3) * kKVHalf + sw128(row, ch & 7);
-          *reinterpret_cast<uint4*>(kst + off) = kv;
-          *reinterpret_cast<uint4*>(kst + 2 * kKVHalf + off) = vv;
+        // tail tile: tokens tb .. tb + 63 of the f new ones, by TMA from
+        // k_new / v_new viewed as [B][f][Hkv][128] (tokens >= f read as zero)
+        const int tb = (t - n_pref) * kTileKeys;
+        if (lane == 0) {
+          mbar_arrive_expect_tx(bar(kBarKvFull + st), 4 * kKVHalf);
+          tma_load_4d(kdst, &tm_kn, bar(kBarKvFull + st), 0, h, tb, b);
+          tma_load_4d(kdst + kKVHalf, &tm_kn, bar(kBarKvFull + st), 64, h, tb, b);
+          tma_load_4d(kdst + 2 * kKVHalf, &tm_vn, bar(kBarKvFull + st), 0, h, tb, b);
+          tma_load_4d(kdst + 3 * kKVHalf, &tm_vn, bar(kBarKvFull + st), 64, h, tb, b);
         }
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(bar(kBarKvFull + st));
       }
     }
   } else if (warp == 1) {
@@ -428,13 +430,14 @@ int rectify_row_groups(int g, int f) {
 }
 
 cudaError_t launch_rectify(const CacheView& c, const CUtensorMap& tm_k, const CUtensorMap& tm_v,
-                           const uint16_t* q_new, const uint16_t* k_new, const uint16_t* v_new, int f,
-                           float sm_scale, int splits, float* o_part, float* lse_part, cudaStream_t st) {
+                           const CUtensorMap& tm_kn, const CUtensorMap& tm_vn, const uint16_t* q_new,
+                           const uint16_t* k_new, const uint16_t* v_new, int f, float sm_scale, int splits,
+                           float* o_part, float* lse_part, cudaStream_t st) {
   cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(rectify_kernel), kSmem, 1);
   if (e != cudaSuccess) return e;
   RectArgs a{q_new, k_new, v_new, f, splits, sm_scale * 1.44269504088896340736f, o_part, lse_part};
   const dim3 grid(splits, rectify_row_groups(c.g, f), c.B * c.Hkv);
-  return launch_pdl(rectify_kernel, grid, dim3(kThreads), kSmem, st, tm_k, tm_v, c, a);
+  return launch_pdl(rectify_kernel, grid, dim3(kThreads), kSmem, st, tm_k, tm_v, tm_kn, tm_vn, c, a);
 }
 
 }  // namespace resa

@@ -77,6 +77,25 @@ resa_status_t pool_tensor_map(const resa_cache_t* c, void* base, CUtensorMap* tm
   return r == CUDA_SUCCESS ? RESA_OK : RESA_ERR_CUDA;
 }
 
+// k_new / v_new of a rectification viewed as a 4-D bf16 tensor
+// [B][f][Hkv][128] (innermost first: dim, head, token, sequence); a box is 64
+// dims x 1 head x 64 tokens (one swizzled half of a 64-key tile), tokens past
+// f read as zero.
+resa_status_t new_kv_tensor_map(const resa_cache_t* c, const void* base, int f, CUtensorMap* tm) {
+  EncodeTiledFn enc = encode_fn();
+  if (enc == nullptr) return RESA_ERR_CUDA;
+  const cuuint64_t row = static_cast<cuuint64_t>(c->head_dim) * 2;
+  const cuuint64_t dims[4] = {static_cast<cuuint64_t>(c->head_dim), static_cast<cuuint64_t>(c->num_kv_heads),
+                              static_cast<cuuint64_t>(f), static_cast<cuuint64_t>(c->batch)};
+  const cuuint64_t strides[3] = {row, row * c->num_kv_heads, row * c->num_kv_heads * f};
+  const cuuint32_t box[4] = {64, 1, 64, 1};
+  const cuuint32_t estr[4] = {1, 1, 1, 1};
+  const CUresult r = enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
+                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? RESA_OK : RESA_ERR_CUDA;
+}
+
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 resa_status_t check_cache(const resa_cache_t* c) {
@@ -345,7 +364,10 @@ resa_status_t resa_rectify_attention(const resa_cache_t* cache, const void* q_ne
   float* lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) +
                                              align_up(rows * splits * kHeadDimHost * sizeof(float)));
   const cudaStream_t st = static_cast<cudaStream_t>(stream);
-  cudaError_t e = launch_rectify(view(cache), tk, tv, static_cast<const uint16_t*>(q_new),
+  CUtensorMap tkn, tvn;
+  if ((s = new_kv_tensor_map(cache, k_new, f, &tkn)) != RESA_OK) return s;
+  if ((s = new_kv_tensor_map(cache, v_new, f, &tvn)) != RESA_OK) return s;
+  cudaError_t e = launch_rectify(view(cache), tk, tv, tkn, tvn, static_cast<const uint16_t*>(q_new),
                                  static_cast<const uint16_t*>(k_new), static_cast<const uint16_t*>(v_new), f,
                                  scale_of(cache, params), splits, o_part, lse_part, st);
   if (e == cudaSuccess)

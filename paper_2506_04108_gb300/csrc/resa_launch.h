@@ -72,7 +72,8 @@ cudaError_t launch_merge(const float* o_part, const float* lse_part, int rows, i
 // rectify.cu
 int rectify_row_groups(int g, int f);
 cudaError_t launch_rectify(const CacheView& c, const CUtensorMap& tm_k, const CUtensorMap& tm_v,
-                           const uint16_t* q_new, const uint16_t* k_new, const uint16_t* v_new, int f,
-                           float sm_scale, int splits, float* o_part, float* lse_part, cudaStream_t st);
+                           const CUtensorMap& tm_kn, const CUtensorMap& tm_vn, const uint16_t* q_new,
+                           const uint16_t* k_new, const uint16_t* v_new, int f, float sm_scale, int splits,
+                           float* o_part, float* lse_part, cudaStream_t st);
 
 }  // namespace resa

@@ -140,6 +140,11 @@ WORKLOADS = {
 # the 32K batch-8 workload's geometry and ReSA parameters at these contexts.
 BREAKDOWN_CONTEXTS = (16384, 65536, 262144)
 
+# Chunked dense prefill: prompt lengths and chunk size.
+PREFILL_LENGTHS = (32768, 131072)
+PREFILL_CHUNK = 4096
+PREFILL_SEED = 2506041086
+
 # Rectification-only sweep: f new queries against cached contexts.
 RECTIFY_SWEEP = [(t, f) for t in (16384, 65536, 262144) for f in (16, 32, 64)]
 RECTIFY_SWEEP_SEED = 2506041085

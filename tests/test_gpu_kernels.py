@@ -318,6 +318,50 @@ def test_rectify_matches_oracle(g, Hkv, lens, f):
         assert np.allclose(lse[b], l, atol=2e-3, rtol=0)
 
 
+@pytest.mark.parametrize("L,C", [(1000, 256), (700, 700), (130, 64)])
+def test_chunked_prefill_equals_dense_causal_attention(L, C):
+    """Algorithm 1's prefill in chunks of C tokens: append the chunk's K/V to
+    the cache (block keys built online), then the rectification call with
+    f = C attends the chunk's queries causally to the cached prefix and the
+    chunk itself. Every prompt position must match dense causal attention over
+    the whole prompt, and the block keys the summaries of the whole prompt."""
+    g, Hkv, B = 7, 2, 2
+    gr = synth.rng(95 + C)
+    Ks = [synth.normal_bf16(gr, (Hkv, L, 128)) for _ in range(B)]
+    Vs = [synth.normal_bf16(gr, (Hkv, L, 128)) for _ in range(B)]
+    Qs = [synth.normal_bf16(gr, (L, g * Hkv, 128)) for _ in range(B)]
+    maxb = (L + 15) // 16 + 1
+    empty = [np.zeros((Hkv, 0, 128), dtype=np.uint16)] * B
+    cache = H.make_cache(empty, empty, g * Hkv, maxb)
+    p = resa.params(0.1, 16, 1)
+    ws, nb = H.workspace(cache, 8, 0, C)
+    outs = []
+    for c0 in range(0, L, C):
+        f = min(C, L - c0)
+        kc = np.stack([np.transpose(Ks[b][:, c0:c0 + f], (1, 0, 2)) for b in range(B)])   # [B, f, Hkv, d]
+        vc = np.stack([np.transpose(Vs[b][:, c0:c0 + f], (1, 0, 2)) for b in range(B)])
+        qc = np.stack([Qs[b][c0:c0 + f] for b in range(B)])                                 # [B, f, Hq, d]
+        kd, vd = H.dev_bf16(kc), H.dev_bf16(vc)
+        resa.resa_commit_kv(cache.struct, kd, vd, f, False)
+        out = torch.empty((B, f, g * Hkv, 128), dtype=torch.bfloat16, device="cuda")
+        resa.resa_rectify_attention(cache.struct, H.dev_bf16(qc), kd, vd, f, p, out, None, ws, nb)
+        outs.append(H.host_f64(out))
+    assert resa.resa_read_device_error(cache.struct) == (0, 0)
+    assert cache.seq_lens.cpu().tolist() == [L] * B
+    out = np.concatenate(outs, axis=1)
+    summ = H.host_bits(cache.summaries)
+    for b in range(B):
+        K, V = O.widen_bf16(Ks[b]), O.widen_bf16(Vs[b])
+        kall, vall = np.transpose(K, (1, 0, 2)), np.transpose(V, (1, 0, 2))
+        o, _ = O.rectify_attention(O.widen_bf16(Qs[b]), K[:, :0], V[:, :0], kall, vall, L, 1 / math.sqrt(128))
+        H.check_outputs(out[b], o, f"prefill b{b}")
+        M = (L + 15) // 16
+        for h in range(Hkv):
+            kmin, kmax = O.block_summaries(K[h], 16)
+            assert np.array_equal(O.widen_bf16(summ[b, h, :M, 0]), kmin)
+            assert np.array_equal(O.widen_bf16(summ[b, h, :M, 1]), kmax)
+
+
 @pytest.mark.parametrize("f,T", [(32, 3000), (16, 1500), (64, 1200)])
 def test_rectify_rescale_path(f, T):
     """Keys whose magnitude ramps up along the positions (and log-normal
