@@ -243,6 +243,21 @@ resa_status_t resa_rectify_attention(const resa_cache_t* cache, const void* q_ne
                                      float* lse, void* workspace, size_t workspace_bytes, void* stream);
 
 /*
+ * Continuous batching (requests at different points of their own rectification
+ * period share a batch): resa_commit_kv and resa_rectify_attention restricted
+ * to the sequences b with active[b] != 0. The others are left exactly as they
+ * are: no cache, length or summary change, no output row written, no device
+ * error recorded for them. active: int32 [batch] on the device (NULL = all,
+ * which is what the plain calls do). Everything else is as in the plain calls.
+ */
+resa_status_t resa_commit_kv_active(const resa_cache_t* cache, const int32_t* active, const void* k_new,
+                                    const void* v_new, int32_t n_tokens, int32_t overwrite, void* stream);
+resa_status_t resa_rectify_attention_active(const resa_cache_t* cache, const int32_t* active, const void* q_new,
+                                            const void* k_new, const void* v_new, int32_t f,
+                                            const resa_params_t* params, void* out, float* lse, void* workspace,
+                                            size_t workspace_bytes, void* stream);
+
+/*
  * resa_sparse_decode without a caller workspace. The paper has no counterpart:
  * this entry point exists for callers that cannot allocate device memory --
  * for example a plugin inside a host framework that owns all device memory

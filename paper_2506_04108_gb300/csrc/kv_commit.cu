@@ -51,6 +51,7 @@ __global__ void __launch_bounds__(256) commit_append_kernel(CacheView c, const u
   pdl_launch_dependents();
   pdl_wait();
   const int b = blockIdx.x;
+  if (c.active != nullptr && c.active[b] == 0) return;
   const int T = c.seq_lens[b];
   const int cap = c.max_blocks * kBlock;
   if (T < 0 || T > cap - n) {
@@ -106,6 +107,7 @@ __global__ void __launch_bounds__(256) commit_overwrite_kernel(CacheView c, cons
   pdl_launch_dependents();
   pdl_wait();
   const int b = blockIdx.y;
+  if (c.active != nullptr && c.active[b] == 0) return;
   const int T = c.seq_lens[b];
   const int cap = c.max_blocks * kBlock;
   if (T < n || T > cap) {

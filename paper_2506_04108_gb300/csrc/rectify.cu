@@ -141,8 +141,9 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
   pdl_launch_dependents();
   pdl_wait();
 
-  const int T = c.seq_lens[b];
-  const bool bad = (T < f || T > c.max_blocks * kBlock);
+  const bool inactive = c.active != nullptr && c.active[b] == 0;  // left out: no work, no output row
+  const int T = inactive ? f : c.seq_lens[b];
+  const bool bad = inactive || (T < f || T > c.max_blocks * kBlock);
   const int P = T - f;  // prefix keys from the cache
   const int ntp = bad ? 0 : (P + kTileKeys - 1) / kTileKeys;
   const int per = (ntp + a.splits - 1) / a.splits;
@@ -153,7 +154,7 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
   const int tok_end = min(f, (row0 + MT * kMTile + 7) / 8);
   const int n_tail = (!bad && s == a.splits - 1) ? (tok_end + kTileKeys - 1) / kTileKeys : 0;
   const int n_tiles = n_pref + n_tail;
-  if (bad && tid == 0 && s == 0 && rg == 0) record_error(c.status, RESA_DEV_SEQ_LEN_RANGE, b);
+  if (bad && !inactive && tid == 0 && s == 0 && rg == 0) record_error(c.status, RESA_DEV_SEQ_LEN_RANGE, b);
 
   // Q tile: rows row0 .. row0 + 128 MT - 1, zero for padding rows
   for (int e0 = 0; e0 < MT * kMTile * 16; e0 += 4 * kThreads) {  // four loads in flight per thread

@@ -141,6 +141,7 @@ CacheView view(const resa_cache_t* c) {
   v.seq_lens = c->seq_lens;
   v.summ = static_cast<uint16_t*>(c->summaries);
   v.status = c->device_status;
+  v.active = nullptr;
   return v;
 }
 
@@ -284,18 +285,24 @@ resa_status_t resa_update_summaries(const resa_cache_t* cache, int32_t block_beg
   return e == cudaSuccess ? RESA_OK : RESA_ERR_CUDA;
 }
 
-resa_status_t resa_commit_kv(const resa_cache_t* cache, const void* k_new, const void* v_new, int32_t n_tokens,
-                             int32_t overwrite, void* stream) {
+resa_status_t resa_commit_kv_active(const resa_cache_t* cache, const int32_t* active, const void* k_new,
+                                    const void* v_new, int32_t n_tokens, int32_t overwrite, void* stream) {
   resa_status_t s = check_cache(cache);
   if (s != RESA_OK) return s;
   if (n_tokens < 0 || n_tokens > cache->max_blocks_per_seq * cache->block_size) return RESA_ERR_INVALID_ARG;
   if (overwrite != 0 && overwrite != 1) return RESA_ERR_INVALID_ARG;
   if (n_tokens > 0 && (k_new == nullptr || v_new == nullptr)) return RESA_ERR_INVALID_ARG;
   if (n_tokens > 0 && (!aligned16(k_new) || !aligned16(v_new))) return RESA_ERR_INVALID_ARG;
-  const cudaError_t e = launch_commit(view(cache), static_cast<const uint16_t*>(k_new),
-                                      static_cast<const uint16_t*>(v_new), n_tokens, overwrite == 1,
-                                      static_cast<cudaStream_t>(stream));
+  CacheView v = view(cache);
+  v.active = active;
+  const cudaError_t e = launch_commit(v, static_cast<const uint16_t*>(k_new), static_cast<const uint16_t*>(v_new),
+                                      n_tokens, overwrite == 1, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? RESA_OK : RESA_ERR_CUDA;
+}
+
+resa_status_t resa_commit_kv(const resa_cache_t* cache, const void* k_new, const void* v_new, int32_t n_tokens,
+                             int32_t overwrite, void* stream) {
+  return resa_commit_kv_active(cache, nullptr, k_new, v_new, n_tokens, overwrite, stream);
 }
 
 resa_status_t resa_select_blocks(const resa_cache_t* cache, const void* q, const resa_params_t* params,
@@ -344,9 +351,10 @@ resa_status_t resa_sparse_decode(const resa_cache_t* cache, const void* q, const
   return e == cudaSuccess ? RESA_OK : RESA_ERR_CUDA;
 }
 
-resa_status_t resa_rectify_attention(const resa_cache_t* cache, const void* q_new, const void* k_new,
-                                     const void* v_new, int32_t f, const resa_params_t* params, void* out,
-                                     float* lse, void* workspace, size_t workspace_bytes, void* stream) {
+resa_status_t resa_rectify_attention_active(const resa_cache_t* cache, const int32_t* active, const void* q_new,
+                                            const void* k_new, const void* v_new, int32_t f,
+                                            const resa_params_t* params, void* out, float* lse, void* workspace,
+                                            size_t workspace_bytes, void* stream) {
   resa_status_t s = check_cache(cache);
   if (s != RESA_OK) return s;
   if ((s = check_params(params)) != RESA_OK) return s;
@@ -367,12 +375,22 @@ resa_status_t resa_rectify_attention(const resa_cache_t* cache, const void* q_ne
   CUtensorMap tkn, tvn;
   if ((s = new_kv_tensor_map(cache, k_new, f, &tkn)) != RESA_OK) return s;
   if ((s = new_kv_tensor_map(cache, v_new, f, &tvn)) != RESA_OK) return s;
-  cudaError_t e = launch_rectify(view(cache), tk, tv, tkn, tvn, static_cast<const uint16_t*>(q_new),
+  CacheView v = view(cache);
+  v.active = active;
+  cudaError_t e = launch_rectify(v, tk, tv, tkn, tvn, static_cast<const uint16_t*>(q_new),
                                  static_cast<const uint16_t*>(k_new), static_cast<const uint16_t*>(v_new), f,
                                  scale_of(cache, params), splits, o_part, lse_part, st);
   if (e == cudaSuccess)
-    e = launch_merge(o_part, lse_part, static_cast<int>(rows), splits, static_cast<uint16_t*>(out), lse, st);
+    e = launch_merge(o_part, lse_part, static_cast<int>(rows), splits, static_cast<uint16_t*>(out), lse, st, active,
+                     f * cache->num_q_heads);
   return e == cudaSuccess ? RESA_OK : RESA_ERR_CUDA;
+}
+
+resa_status_t resa_rectify_attention(const resa_cache_t* cache, const void* q_new, const void* k_new,
+                                     const void* v_new, int32_t f, const resa_params_t* params, void* out,
+                                     float* lse, void* workspace, size_t workspace_bytes, void* stream) {
+  return resa_rectify_attention_active(cache, nullptr, q_new, k_new, v_new, f, params, out, lse, workspace,
+                                       workspace_bytes, stream);
 }
 
 }  // extern "C"

@@ -25,6 +25,7 @@ struct CacheView {
   int32_t* seq_lens;
   uint16_t* summ;
   int32_t* status;
+  const int32_t* active;  // [B]: sequences with 0 are left out of commits and rectification; null = all
 };
 
 // Launches `kernel` with programmatic stream serialization (see
@@ -67,7 +68,7 @@ cudaError_t launch_sparse_decode(const CacheView& c, const CUtensorMap& tm_k, co
                                  const uint16_t* q, const int32_t* indices, const int32_t* counts, int n_cap,
                                  float sm_scale, int splits, float* o_part, float* lse_part, cudaStream_t st);
 cudaError_t launch_merge(const float* o_part, const float* lse_part, int rows, int splits, uint16_t* out,
-                         float* lse_out, cudaStream_t st);
+                         float* lse_out, cudaStream_t st, const int32_t* active = nullptr, int rows_per_seq = 1);
 
 // rectify.cu
 int rectify_row_groups(int g, int f);

@@ -299,11 +299,14 @@ constexpr int kMergeWarps = 8;
 __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const float* __restrict__ o_part,
                                                                  const float* __restrict__ lse_part, int splits,
                                                                  uint16_t* __restrict__ out,
-                                                                 float* __restrict__ lse_out) {
+                                                                 float* __restrict__ lse_out,
+                                                                 const int32_t* __restrict__ active,
+                                                                 int rows_per_seq) {
   __shared__ float4 red[kMergeWarps][kHeadDim / 4];
   pdl_launch_dependents();
   pdl_wait();
   const size_t row = blockIdx.x;
+  if (active != nullptr && active[row / rows_per_seq] == 0) return;  // a sequence left out of the call
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const float* lp = lse_part + row * splits;
   float m = kNegInf;
@@ -382,10 +385,10 @@ cudaError_t launch_sparse_decode(const CacheView& c, const CUtensorMap& tm_k, co
 }
 
 cudaError_t launch_merge(const float* o_part, const float* lse_part, int rows, int splits, uint16_t* out,
-                         float* lse_out, cudaStream_t st) {
+                         float* lse_out, cudaStream_t st, const int32_t* active, int rows_per_seq) {
   if (rows == 0) return cudaSuccess;
   return launch_pdl(merge_kernel, dim3(rows), dim3(kMergeWarps * 32), 0, st, o_part, lse_part, splits, out,
-                    lse_out);
+                    lse_out, active, rows_per_seq);
 }
 
 }  // namespace resa

@@ -26,7 +26,8 @@ DEVICE_ERRORS = {0: "RESA_DEV_OK", 1: "RESA_DEV_SEQ_LEN_RANGE", 2: "RESA_DEV_PAG
                  3: "RESA_DEV_BUDGET_OVER_CAP", 4: "RESA_DEV_WAIT_TIMEOUT", 5: "RESA_DEV_BAD_INDEX"}
 EXPORTED = ["resa_abi_version", "resa_status_string", "resa_max_selected", "resa_decode_num_splits",
             "resa_workspace_size", "resa_update_summaries", "resa_commit_kv", "resa_select_blocks",
-            "resa_sparse_decode", "resa_rectify_attention", "resa_read_device_error", "resa_sparse_decode_static"]
+            "resa_sparse_decode", "resa_rectify_attention", "resa_read_device_error", "resa_sparse_decode_static",
+            "resa_commit_kv_active", "resa_rectify_attention_active"]
 
 
 class ResaError(RuntimeError):
@@ -73,6 +74,8 @@ def load() -> ctypes.CDLL:
         "resa_rectify_attention": ([cp, pp, pp, pp, c_int32, pc, pp, pp, pp, c_size_t, pp], c_int32),
         "resa_read_device_error": ([cp, POINTER(c_int32), POINTER(c_int32), pp], c_int32),
         "resa_sparse_decode_static": ([cp, pp, pp, pp, c_int32, pc, pp, pp, c_int32, pp], c_int32),
+        "resa_commit_kv_active": ([cp, pp, pp, pp, c_int32, c_int32, pp], c_int32),
+        "resa_rectify_attention_active": ([cp, pp, pp, pp, pp, c_int32, pc, pp, pp, pp, c_size_t, pp], c_int32),
     }
     for name, (args, ret) in sig.items():
         fn = getattr(L, name)
@@ -183,6 +186,22 @@ def resa_read_device_error(cache: ResaCacheT, stream=None) -> tuple[int, int]:
     if st not in (RESA_OK, 5):
         raise ResaError(st, "resa_read_device_error")
     return code.value, detail.value
+
+
+def resa_commit_kv_active(cache: ResaCacheT, active, k_new, v_new, n_tokens: int, overwrite: bool, stream=None):
+    """resa_commit_kv for the sequences with active[b] != 0 only (continuous batching)."""
+    _check(load().resa_commit_kv_active(ctypes.byref(cache), _ptr(active), _ptr(k_new), _ptr(v_new), n_tokens,
+                                        int(bool(overwrite)), _stream(stream)), "resa_commit_kv_active")
+
+
+def resa_rectify_attention_active(cache: ResaCacheT, active, q_new, k_new, v_new, f: int, p: ResaParamsT, out, lse,
+                                  workspace, workspace_bytes: int, stream=None):
+    """resa_rectify_attention for the sequences with active[b] != 0 only; the
+    output rows of the others are not written."""
+    _check(load().resa_rectify_attention_active(ctypes.byref(cache), _ptr(active), _ptr(q_new), _ptr(k_new),
+                                                _ptr(v_new), f, ctypes.byref(p), _ptr(out), _ptr(lse),
+                                                _ptr(workspace), workspace_bytes, _stream(stream)),
+           "resa_rectify_attention_active")
 
 
 # ------------------------------------------------------ caller buffers ---

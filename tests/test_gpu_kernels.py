@@ -362,6 +362,54 @@ def test_chunked_prefill_equals_dense_causal_attention(L, C):
             assert np.array_equal(O.widen_bf16(summ[b, h, :M, 1]), kmax)
 
 
+def test_active_mask_commit_and_rectify():
+    """Continuous batching: only sequences with active[b] != 0 are rectified,
+    appended to or overwritten; the others keep their cache, length, block
+    keys and output rows, and record no error."""
+    g, Hkv, f = 4, 2, 16
+    lens = [700, 333, 1025]
+    B = len(lens)
+    Ks, Vs = seq_inputs(97, B, Hkv, lens)
+    maxb = max((T + 15) // 16 for T in lens) + 4
+    cache = H.make_cache(Ks, Vs, g * Hkv, maxb)
+    active = torch.tensor([1, 0, 1], dtype=torch.int32, device="cuda")
+    gr = synth.rng(98)
+    qn = synth.normal_bf16(gr, (B, f, g * Hkv, 128))
+    kn = synth.normal_bf16(gr, (B, f, Hkv, 128))
+    vn = synth.normal_bf16(gr, (B, f, Hkv, 128))
+    p = resa.params(0.1, 16, 1)
+    ws, nb = H.workspace(cache, 8, 0, f)
+    out = torch.full((B, f, g * Hkv, 128), 7.0, dtype=torch.bfloat16, device="cuda")
+    resa.resa_rectify_attention_active(cache.struct, active, H.dev_bf16(qn), H.dev_bf16(kn), H.dev_bf16(vn), f, p,
+                                       out, None, ws, nb)
+    assert resa.resa_read_device_error(cache.struct) == (0, 0)
+    o_host = H.host_f64(out)
+    assert np.all(o_host[1] == 7.0)                      # left out: untouched
+    for b in (0, 2):
+        o, _ = O.rectify_attention(O.widen_bf16(qn[b]), O.widen_bf16(Ks[b]), O.widen_bf16(Vs[b]),
+                                   O.widen_bf16(kn[b]), O.widen_bf16(vn[b]), lens[b], 1 / math.sqrt(128))
+        H.check_outputs(o_host[b], o, f"rectify active b{b}")
+    # overwrite commit of the f tokens: the left-out sequence keeps its K/V and block keys
+    kp0, sm0 = H.host_bits(cache.k_pool).copy(), H.host_bits(cache.summaries).copy()
+    resa.resa_commit_kv_active(cache.struct, active, H.dev_bf16(kn), H.dev_bf16(vn), f, True)
+    assert resa.resa_read_device_error(cache.struct) == (0, 0)
+    sm1 = H.host_bits(cache.summaries)
+    assert np.array_equal(sm1[1], sm0[1])
+    for b in (0, 2):
+        K, _ = H.logical_kv(cache, b)
+        assert np.array_equal(np.transpose(K[:, lens[b] - f:], (1, 0, 2)), kn[b])
+        kmin, kmax = O.block_summaries(O.widen_bf16(K[0]), 16)
+        M = (lens[b] + 15) // 16
+        assert np.array_equal(O.widen_bf16(sm1[b, 0, :M, 0]), kmin)
+    K1, _ = H.logical_kv(cache, 1)
+    assert np.array_equal(K1, Ks[1])
+    # append of 3 tokens: only active sequences grow
+    ka = synth.normal_bf16(gr, (B, 3, Hkv, 128))
+    resa.resa_commit_kv_active(cache.struct, active, H.dev_bf16(ka), H.dev_bf16(ka), 3, False)
+    assert cache.seq_lens.cpu().tolist() == [lens[0] + 3, lens[1], lens[2] + 3]
+    assert resa.resa_read_device_error(cache.struct) == (0, 0)
+
+
 @pytest.mark.parametrize("f,T", [(32, 3000), (16, 1500), (64, 1200)])
 def test_rectify_rescale_path(f, T):
     """Keys whose magnitude ramps up along the positions (and log-normal
