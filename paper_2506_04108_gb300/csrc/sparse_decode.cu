@@ -290,11 +290,13 @@ __global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid
   }
 }
 
-// One CTA of 8 warps per output row: every warp reduces the split
-// log2-sum-exps itself (shuffles, no barrier), then warp w accumulates the
-// splits w, w + 8, ... for 4 of the 128 dims per lane, four splits' loads in
-// flight at a time; the 8 partial rows are summed through shared memory.
+// One CTA of 8 warps per output row. Warp w takes the splits w, w + 8, ...:
+// its lanes load ten partial rows (16 bytes each) and their log2-sum-exps at
+// once, so up to 80 splits cost one round of loads; each warp keeps its sum
+// relative to its own maximum, and the warps' maxima and rows are combined
+// through shared memory.
 constexpr int kMergeWarps = 8;
+constexpr int kMergeLoads = 10;  // partial rows in flight per lane (80 splits in one round)
 
 __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const float* __restrict__ o_part,
                                                                  const float* __restrict__ lse_part, int splits,
@@ -303,41 +305,54 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const float* __
                                                                  const int32_t* __restrict__ active,
                                                                  int rows_per_seq) {
   __shared__ float4 red[kMergeWarps][kHeadDim / 4];
+  __shared__ float wmax[kMergeWarps];
   pdl_launch_dependents();
   pdl_wait();
   const size_t row = blockIdx.x;
   if (active != nullptr && active[row / rows_per_seq] == 0) return;  // a sequence left out of the call
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const float* lp = lse_part + row * splits;
-  float m = kNegInf;
-  for (int s = lane; s < splits; s += 32) m = fmaxf(m, lp[s]);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-  const float base = safe_base(m);
-  float l = 0.f;
-  for (int s = lane; s < splits; s += 32) l += exp2f(lp[s] - base);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
   const float4* op = reinterpret_cast<const float4*>(o_part + row * splits * kHeadDim) + lane;
+  // this warp's splits w + 8 j and their log2-sum-exps, ten of each in
+  // flight together (one pass for up to 80 splits, an online rescale beyond)
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  for (int s0 = warp; s0 < splits; s0 += 4 * kMergeWarps) {
-    float4 v[4];
-    float w[4];
+  float m = kNegInf;
+  for (int base = 0; base < splits; base += kMergeWarps * kMergeLoads) {
+    float4 v[kMergeLoads];
+    float ls[kMergeLoads];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int s = s0 + u * kMergeWarps;
-      const bool ok = s < splits;
-      v[u] = ok ? op[s * (kHeadDim / 4)] : make_float4(0.f, 0.f, 0.f, 0.f);
-      w[u] = ok ? exp2f(lp[s] - base) : 0.f;
+    for (int j = 0; j < kMergeLoads; ++j) {
+      const int sp = base + warp + kMergeWarps * j;
+      const bool ok = sp < splits;
+      v[j] = ok ? op[static_cast<size_t>(sp) * (kHeadDim / 4)] : make_float4(0.f, 0.f, 0.f, 0.f);
+      ls[j] = ok ? lp[sp] : kNegInf;
     }
+    float mb = m;
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      acc.x += w[u] * v[u].x;
-      acc.y += w[u] * v[u].y;
-      acc.z += w[u] * v[u].z;
-      acc.w += w[u] * v[u].w;
+    for (int j = 0; j < kMergeLoads; ++j) mb = fmaxf(mb, ls[j]);
+    const float sc = m == kNegInf ? 0.f : exp2f(m - safe_base(mb));
+    acc.x *= sc;
+    acc.y *= sc;
+    acc.z *= sc;
+    acc.w *= sc;
+    m = mb;
+#pragma unroll
+    for (int j = 0; j < kMergeLoads; ++j) {
+      const float w = exp2f(ls[j] - safe_base(m));
+      acc.x += w * v[j].x;
+      acc.y += w * v[j].y;
+      acc.z += w * v[j].z;
+      acc.w += w * v[j].w;
     }
   }
+  // acc is this warp's sum relative to its own maximum m: rescale to the CTA's
+  if (lane == 0) wmax[warp] = m;
+  __syncthreads();
+  float M = kNegInf;
+#pragma unroll
+  for (int w = 0; w < kMergeWarps; ++w) M = fmaxf(M, wmax[w]);
+  const float sc = m == kNegInf ? 0.f : exp2f(m - safe_base(M));
+  acc.x *= sc; acc.y *= sc; acc.z *= sc; acc.w *= sc;
   red[warp][lane] = acc;
   __syncthreads();
   if (warp == 0) {
@@ -349,12 +364,17 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const float* __
       t.z += red[w][lane].z;
       t.w += red[w][lane].w;
     }
+    // the normaliser: sum over all splits of exp2(lse - M), lane-strided
+    float l = 0.f;
+    for (int sp = lane; sp < splits; sp += 32) l += exp2f(lp[sp] - safe_base(M));
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
     const float inv = l > 0.f ? 1.f / l : 0.f;
     uint2 packed;
     packed.x = pack_bf16x2(t.x * inv, t.y * inv);
     packed.y = pack_bf16x2(t.z * inv, t.w * inv);
     *reinterpret_cast<uint2*>(out + row * kHeadDim + 4 * lane) = packed;
-    if (lse_out != nullptr && lane == 0) lse_out[row] = l > 0.f ? (m + log2f(l)) * 0.69314718055994530942f : kNegInf;
+    if (lse_out != nullptr && lane == 0) lse_out[row] = l > 0.f ? (M + log2f(l)) * 0.69314718055994530942f : kNegInf;
   }
 }
 
