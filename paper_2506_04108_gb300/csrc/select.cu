@@ -7,17 +7,23 @@
 //               half-warp takes one block, a lane one 16-byte piece (8 dims)
 //               of k_min and k_max, and the 128-dim sum is a fixed-order
 //               butterfly over the 16 lanes.
-// topn_kernel   one 8-CTA cluster per (sequence, KV head). The n of Eq. 5 is
-//               evaluated on the device from the device-resident length. The
-//               last n_local blocks are always taken (score +inf); the rest
-//               of the budget is the largest order-preserving keys of the
-//               other blocks, found by a radix select over key - min key with
-//               8-bit digits from the top significant bit of the unit's key
-//               range (keys staged in the CTAs' shared memory, histograms
-//               summed across the cluster through distributed shared memory).
-//               The selected ids are written in ascending order by a ballot
-//               compaction that resolves ties at the threshold toward the
-//               lower block index.
+// top-n        one CTA (caches of up to kTopnCtaMaxBlocks blocks per
+//               sequence) or one 8-CTA cluster (larger caches) per (sequence,
+//               KV head). The n of Eq. 5 is evaluated on the device from the
+//               device-resident length. The last n_local blocks are always
+//               taken (score +inf); the rest of the budget is the largest
+//               order-preserving keys of the other blocks, found by a radix
+//               select over key - min key with 8-bit digits from the top
+//               significant bit of the unit's key range (keys staged in shared
+//               memory; in the cluster form the histograms are summed across
+//               the cluster through distributed shared memory). The selected
+//               ids are written in ascending order by a ballot compaction that
+//               resolves ties at the threshold toward the lower block index.
+//
+// Both top-n kernels read the length and evaluate Eq. 5 before waiting on the
+// score kernel: that kernel lets its dependents launch only after its own wait
+// on the preceding kernel (the append commit that advances the length) has
+// returned, and the length is read from L2.
 #include <cooperative_groups.h>
 
 #include <atomic>
@@ -32,6 +38,10 @@ constexpr int kTopnCluster = 8;                                   // CTAs per (s
 constexpr int kTopnThreads = 256;
 constexpr int kTopnWarps = kTopnThreads / 32;
 constexpr int kTopnSmemMax = 200 * 1024;                           // staged keys per CTA, bytes
+constexpr int kTopnCtaThreads = 512;                                // one-CTA form
+constexpr int kTopnCtaWarps = kTopnCtaThreads / 32;
+constexpr int kTopnCtaMaxBlocks = 6144;  // the one-CTA form serves caches up to this many blocks per sequence
+static_assert(kTopnCtaMaxBlocks * sizeof(uint32_t) <= 48 * 1024, "one-CTA top-n keys fit the default shared memory");
 
 // Exact max of two packed bf16 pairs.
 __device__ __forceinline__ uint32_t bf16x2_max(uint32_t a, uint32_t b) {
@@ -131,7 +141,6 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c,
     blk0 = (r % per_head) * kPieceBlocks;
     nblk = min(kPieceBlocks, M - blk0);
   };
-  pdl_launch_dependents();
   // Before the wait for the preceding kernel, prefetch this warp's pieces into
   // L2 from the lengths as they are now (the append commit that may still be
   // running changes at most the last block of a sequence; a stale length only
@@ -153,6 +162,9 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c,
   }
   __syncthreads();  // the tables are rebuilt below
   pdl_wait();
+  // The top-n kernel reads the lengths before its own wait: let it launch
+  // only now that the append commit (which advances them) has completed.
+  pdl_launch_dependents();
   build_tables();
   const int total = sh_pref[c.B];
   const int per = (total + gridDim.x - 1) / gridDim.x;
@@ -256,6 +268,32 @@ __device__ __forceinline__ uint32_t score_key(float s) {
   return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
+// Eq. 5 for one unit: n = max(n_min, ceil(M keep)), at least n_local and at
+// most M, clamped to the id row's capacity (reported). Blocks [F, M) are the
+// forced local blocks (score +inf), nf of them taken; r blocks are picked
+// among [0, F).
+struct UnitBudget {
+  int M, n, F, nf, r;
+};
+__device__ __forceinline__ UnitBudget unit_budget(int T, double keep, int n_min, int n_local, int n_cap,
+                                                  int32_t* status, int unit, bool report) {
+  UnitBudget u;
+  u.M = (T + kBlock - 1) / kBlock;
+  long long nn = static_cast<long long>(ceil(static_cast<double>(u.M) * keep));
+  nn = max(nn, static_cast<long long>(n_min));
+  nn = max(nn, static_cast<long long>(n_local));
+  nn = min(nn, static_cast<long long>(u.M));
+  u.n = static_cast<int>(nn);
+  if (u.n > n_cap) {
+    if (report) record_error(status, RESA_DEV_BUDGET_OVER_CAP, unit);
+    u.n = n_cap;
+  }
+  u.F = u.M - min(n_local, u.M);
+  u.nf = min(u.M - u.F, u.n);
+  u.r = u.n - u.nf;
+  return u;
+}
+
 // Exclusive scan of one int per warp (kTopnWarps values, in place) by warp 0.
 __device__ __forceinline__ void scan_warp_totals(int* vals) {
   const int lane = threadIdx.x & 31;
@@ -295,12 +333,12 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
   namespace cg = cooperative_groups;
   cg::cluster_group cluster = cg::this_cluster();
   pdl_launch_dependents();
-  pdl_wait();
   const int rank = static_cast<int>(cluster.block_rank());
   const int b = blockIdx.z, h = blockIdx.y;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   int32_t* out = indices + (static_cast<size_t>(b) * c.Hkv + h) * n_cap;
-  const int T = c.seq_lens[b];
+  const int T = __ldcg(c.seq_lens + b);  // final before the score kernel let this one launch
+  pdl_wait();                            // the scores
   if (T < 0 || T > c.max_blocks * kBlock) {  // the whole cluster takes this branch
     if (rank == 0 && tid == 0) {
       record_error(c.status, RESA_DEV_SEQ_LEN_RANGE, b);
@@ -309,24 +347,12 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
     for (int i = rank * kTopnThreads + tid; i < n_cap; i += kTopnCluster * kTopnThreads) out[i] = -1;
     return;
   }
-  const int M = (T + kBlock - 1) / kBlock;
-  // Eq. 5 on the device: n = max(n_min, ceil(M * keep)), n_local <= n <= M
-  long long nn = static_cast<long long>(ceil(static_cast<double>(M) * keep));
-  nn = max(nn, static_cast<long long>(n_min));
-  nn = max(nn, static_cast<long long>(n_local));
-  nn = min(nn, static_cast<long long>(M));
-  int n = static_cast<int>(nn);
-  if (n > n_cap) {
-    if (rank == 0 && tid == 0) record_error(c.status, RESA_DEV_BUDGET_OVER_CAP, b * c.Hkv + h);
-    n = n_cap;
-  }
+  const UnitBudget u = unit_budget(T, keep, n_min, n_local, n_cap, c.status, b * c.Hkv + h, rank == 0 && tid == 0);
+  const int M = u.M, n = u.n, F = u.F, nf = u.nf, r = u.r;
   const int per = (M + kTopnCluster - 1) / kTopnCluster;
   const int lo = rank * per, cnt = max(0, min(M, lo + per) - lo);
   const float* sc = scores + (static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks + lo;
-  const int F = M - min(n_local, M);  // blocks [F, M) are forced (score +inf)
-  const int nf = min(M - F, n);       // forced blocks taken (all unless n was clamped)
-  const int r = n - nf;               // blocks to pick among [0, F)
-  const int f_loc = F - lo;           // this CTA's ids >= f_loc are forced
+  const int f_loc = F - lo;  // this CTA's ids >= f_loc are forced
   uint32_t kmin = 0xFFFFFFFFu, kmax = 0u;
   for (int i0 = 0; i0 < cnt; i0 += 4 * kTopnThreads) {  // four loads in flight per thread
     float v[4];
@@ -532,9 +558,202 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
   cluster.sync();  // no CTA leaves while a peer may still read its counts
 }
 
+
+// One-CTA radix select, grid (KV head, sequence), for caches of up to
+// kTopnCtaMaxBlocks blocks per sequence: the same selection as topn_kernel
+// with every barrier a CTA barrier. The histograms rotate through three
+// buffers, so one barrier per pass suffices (the buffer zeroed during a pass
+// was last read two passes before); warp 0 finds each digit and one more
+// barrier hands it to the other warps. The ordered compaction gives each warp
+// a contiguous id range, and every warp derives its output offset from the
+// per-warp counts after a single barrier.
+__global__ void __launch_bounds__(kTopnCtaThreads, 1) topn_cta_kernel(CacheView c, const float* __restrict__ scores,
+                                                                      double keep, int n_min, int n_local,
+                                                                      int32_t* __restrict__ indices,
+                                                                      int32_t* __restrict__ counts, int n_cap) {
+  extern __shared__ uint32_t keys[];
+  __shared__ __align__(16) int hist[3][256];
+  __shared__ uint32_t w_lo[kTopnCtaWarps], w_hi[kTopnCtaWarps];
+  __shared__ int w_gt[kTopnCtaWarps], w_eq[kTopnCtaWarps];
+  __shared__ int sh_pick[3];  // digit, rank left, whole bucket taken
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (int i = tid; i < 2 * 256; i += kTopnCtaThreads) (&hist[0][0])[i] = 0;
+  pdl_launch_dependents();
+  const int h = blockIdx.x, b = blockIdx.y;
+  int32_t* out = indices + (static_cast<size_t>(b) * c.Hkv + h) * n_cap;
+  const int T = __ldcg(c.seq_lens + b);  // final before the score kernel let this one launch
+  if (T < 0 || T > c.max_blocks * kBlock) {
+    pdl_wait();
+    if (tid == 0) {
+      record_error(c.status, RESA_DEV_SEQ_LEN_RANGE, b);
+      counts[b * c.Hkv + h] = 0;
+    }
+    for (int i = tid; i < n_cap; i += kTopnCtaThreads) out[i] = -1;
+    return;
+  }
+  const UnitBudget u = unit_budget(T, keep, n_min, n_local, n_cap, c.status, b * c.Hkv + h, tid == 0);
+  const int M = u.M, n = u.n, F = u.F, nf = u.nf, r = u.r;
+  const float* sc = scores + (static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks;
+  pdl_wait();  // the scores
+  uint32_t kmin = 0xFFFFFFFFu, kmax = 0u;
+  for (int i0 = 0; i0 < M; i0 += 4 * kTopnCtaThreads) {  // four loads in flight per thread
+    float v[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int i = i0 + k * kTopnCtaThreads + tid;
+      v[k] = i < M ? sc[i] : 0.f;
+    }
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int i = i0 + k * kTopnCtaThreads + tid;
+      if (i < M) {
+        const uint32_t key = score_key(v[k]);
+        keys[i] = key;
+        if (i < F) {
+          kmin = min(kmin, key);
+          kmax = max(kmax, key);
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    kmin = min(kmin, __shfl_xor_sync(0xffffffffu, kmin, o));
+    kmax = max(kmax, __shfl_xor_sync(0xffffffffu, kmax, o));
+  }
+  if (lane == 0) {
+    w_lo[warp] = kmin;
+    w_hi[warp] = kmax;
+  }
+  __syncthreads();  // the keys and the per-warp extremes are visible
+  kmin = lane < kTopnCtaWarps ? w_lo[lane] : 0xFFFFFFFFu;
+  kmax = lane < kTopnCtaWarps ? w_hi[lane] : 0u;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    kmin = min(kmin, __shfl_xor_sync(0xffffffffu, kmin, o));
+    kmax = max(kmax, __shfl_xor_sync(0xffffffffu, kmax, o));
+  }
+
+  // ---- radix select of the r-th largest v = key - kmin among blocks [0, F) ----
+  uint32_t prefix = 0, pmask = 0;
+  int rem = r;
+  if (r > 0 && r < F) {
+    const int bits = 32 - __clz(static_cast<int>(kmax - kmin));  // significant bits of v
+    int shift = max(bits - 8, 0), width = bits - shift;
+    for (int pass = 0;; ++pass) {
+      const uint32_t dmask = (1u << width) - 1u;
+      int* hb = hist[pass % 3];
+      for (int i = tid; i < 256; i += kTopnCtaThreads) hist[(pass + 1) % 3][i] = 0;
+      for (int i = tid; i < F; i += kTopnCtaThreads) {
+        const uint32_t v = keys[i] - kmin;
+        if ((v & pmask) == prefix) atomicAdd(&hb[(v >> shift) & dmask], 1);
+      }
+      __syncthreads();  // this pass's histogram is complete
+      if (warp == 0) {
+        // lane l owns digits 255-8l ... 248-8l (descending): two 16-byte loads
+        const int4 a0 = reinterpret_cast<const int4*>(hb)[2 * (31 - lane)];
+        const int4 a1 = reinterpret_cast<const int4*>(hb)[2 * (31 - lane) + 1];
+        const int cn[8] = {a1.w, a1.z, a1.y, a1.x, a0.w, a0.z, a0.y, a0.x};
+        int sum = 0;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) sum += cn[j];
+        int incl = sum;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int y = __shfl_up_sync(0xffffffffu, incl, o);
+          if (lane >= o) incl += y;
+        }
+        const int excl = incl - sum;
+        if (excl < rem && rem <= incl) {
+          int cum = excl;
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            if (cum + cn[j] >= rem) {
+              sh_pick[0] = 255 - 8 * lane - j;
+              sh_pick[1] = rem - cum;
+              sh_pick[2] = (rem - cum == cn[j]) ? 1 : 0;  // the whole bucket is taken
+              break;
+            }
+            cum += cn[j];
+          }
+        }
+      }
+      __syncthreads();  // the digit is visible
+      prefix |= static_cast<uint32_t>(sh_pick[0]) << shift;
+      pmask |= dmask << shift;
+      rem = sh_pick[1];
+      if (sh_pick[2] || shift == 0) break;
+      width = min(8, shift);
+      shift -= width;
+    }
+  }
+  // Selected: forced blocks [F, F + nf), and among [0, F) the ids with
+  // (v & pmask) > prefix, or == prefix among the first `take_eq` such ids.
+  const int take_eq = rem;
+  auto classify = [&](int i, bool in, bool& is_gt, bool& is_eq) {
+    is_gt = false;
+    is_eq = false;
+    if (in) {
+      if (i >= F) {
+        is_gt = i - F < nf;
+      } else {
+        const uint32_t v = (keys[i] - kmin) & pmask;
+        is_gt = v > prefix;
+        is_eq = v == prefix;
+      }
+    }
+  };
+  const int per_warp = ((M + 31) / 32 + kTopnCtaWarps - 1) / kTopnCtaWarps * 32;
+  const int w0 = warp * per_warp, w1 = min(M, w0 + per_warp);
+  int gt = 0, eq = 0;
+  for (int i0 = w0; i0 < w1; i0 += 32) {
+    bool is_gt, is_eq;
+    classify(i0 + lane, i0 + lane < w1, is_gt, is_eq);
+    gt += __popc(__ballot_sync(0xffffffffu, is_gt));
+    eq += __popc(__ballot_sync(0xffffffffu, is_eq));
+  }
+  if (lane == 0) {
+    w_gt[warp] = gt;
+    w_eq[warp] = eq;
+  }
+  __syncthreads();  // every warp's counts are visible
+  // this warp's offsets: equal keys and selected ids of the lower warps
+  const int e_l = lane < kTopnCtaWarps ? w_eq[lane] : 0, g_l = lane < kTopnCtaWarps ? w_gt[lane] : 0;
+  int ie = e_l;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, ie, o);
+    if (lane >= o) ie += y;
+  }
+  const int s_l = g_l + max(0, min(e_l, take_eq - (ie - e_l)));
+  int is = s_l;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, is, o);
+    if (lane >= o) is += y;
+  }
+  int eq_seen = __shfl_sync(0xffffffffu, ie - e_l, warp);
+  int pos = __shfl_sync(0xffffffffu, is - s_l, warp);
+  for (int i0 = w0; i0 < w1; i0 += 32) {
+    const int i = i0 + lane;
+    bool is_gt, is_eq;
+    classify(i, i < w1, is_gt, is_eq);
+    const unsigned eqm = __ballot_sync(0xffffffffu, is_eq);
+    const int my_eq_rank = eq_seen + __popc(eqm & ((1u << lane) - 1u));
+    const bool sel = is_gt || (is_eq && my_eq_rank < take_eq);
+    const unsigned selm = __ballot_sync(0xffffffffu, sel);
+    if (sel) out[pos + __popc(selm & ((1u << lane) - 1u))] = i;
+    eq_seen += __popc(eqm);
+    pos += __popc(selm);
+  }
+  for (int i = n + tid; i < n_cap; i += kTopnCtaThreads) out[i] = -1;
+  if (tid == 0) counts[b * c.Hkv + h] = n;
+}
+
 }  // namespace
 
 size_t select_smem_bytes(int max_blocks) {
+  if (max_blocks <= kTopnCtaMaxBlocks) return static_cast<size_t>(max_blocks) * sizeof(uint32_t);
   return static_cast<size_t>((max_blocks + kTopnCluster - 1) / kTopnCluster) * sizeof(uint32_t);
 }
 
@@ -552,6 +771,9 @@ cudaError_t launch_select(const CacheView& c, const uint16_t* q, double keep, in
   e = launch_pdl(score_kernel, dim3(grid), dim3(kScoreWarps * 32), kScoreSmem, st, c, q, scores);
   if (e != cudaSuccess) return e;
   const size_t smem = select_smem_bytes(c.max_blocks);
+  if (c.max_blocks <= kTopnCtaMaxBlocks)
+    return launch_pdl(topn_cta_kernel, dim3(c.Hkv, c.B), dim3(kTopnCtaThreads), smem, st, c,
+                      static_cast<const float*>(scores), keep, n_min, n_local, indices, counts, n_cap);
   if (smem > 48 * 1024) {
     e = ensure_smem_attr(reinterpret_cast<const void*>(topn_kernel), kTopnSmemMax, 2);
     if (e != cudaSuccess) return e;

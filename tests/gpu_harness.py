@@ -27,13 +27,24 @@ def host_f64(t: torch.Tensor) -> np.ndarray:
     return O.widen_bf16(host_bits(t))
 
 
-def make_cache(Ks, Vs, Hq, max_blocks, seed=1, zero_pools=False):
+def make_cache(Ks, Vs, Hq, max_blocks, seed=1, zero_pools=False, compact=False):
     """Paged cache holding per-sequence keys/values Ks[b], Vs[b] (uint16 bits,
     [Hkv, T_b, d]; ragged T_b allowed), pages scattered by a seeded page table.
-    Summaries are built with resa_update_summaries."""
+    Summaries are built with resa_update_summaries. `compact` gives pages only
+    to the blocks the sequences hold (the rest of each page-table row points at
+    page 0): for wide page-table rows whose tail is never touched."""
     B = len(Ks)
     Hkv = Ks[0].shape[0]
-    pt = synth.page_table(synth.rng(seed), B, max_blocks)
+    if compact:
+        need = [(K.shape[1] + 15) // 16 for K in Ks]
+        perm = synth.rng(seed).permutation(max(1, sum(need))).astype(np.int32)
+        pt = np.zeros((B, max_blocks), dtype=np.int32)
+        off = 0
+        for b, m in enumerate(need):
+            pt[b, :m] = perm[off:off + m]
+            off += m
+    else:
+        pt = synth.page_table(synth.rng(seed), B, max_blocks)
     cache = resa.PagedKVCache(B, Hq, Hkv, max_blocks, pt, zero_pools=zero_pools)
     kp = host_bits(cache.k_pool).copy()
     vp = host_bits(cache.v_pool).copy()

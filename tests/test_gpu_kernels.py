@@ -105,6 +105,10 @@ def run_select(cache, q_bits, p, n_cap):
     return idx.cpu().numpy(), cnt.cpu().numpy()
 
 
+# Caches of up to 6144 blocks per sequence take the one-CTA top-n, larger ones
+# the cluster top-n: `wide` pads the page-table row past that bound so that
+# every case runs through both.
+@pytest.mark.parametrize("wide", [False, True])
 @pytest.mark.parametrize("g,Hkv,lens,keep,n_min,n_local", [
     (4, 2, [4100], 0.1, 16, 4),            # the 4K workload shape
     (7, 4, [1000, 2053, 37, 16], 0.1, 8, 1),
@@ -113,10 +117,12 @@ def run_select(cache, q_bits, p, n_cap):
     (7, 4, [100, 80], 0.5, 16, 1),         # M <= n: every block selected
     (2, 2, [160], 0.0, 0, 12),             # n_local >= n
 ])
-def test_select_matches_oracle(g, Hkv, lens, keep, n_min, n_local):
+def test_select_matches_oracle(g, Hkv, lens, keep, n_min, n_local, wide):
     Ks, Vs = seq_inputs(5 + len(lens), len(lens), Hkv, lens)
     maxb = max((T + 15) // 16 for T in lens) + 4
-    cache = H.make_cache(Ks, Vs, g * Hkv, maxb)
+    if wide:
+        maxb = max(maxb, 6200)
+    cache = H.make_cache(Ks, Vs, g * Hkv, maxb, compact=wide)
     gq = synth.rng(55)
     q = synth.normal_bf16(gq, (len(lens), g * Hkv, 128))
     p = resa.params(keep, n_min, n_local)
@@ -145,7 +151,8 @@ def check_select_case(cache, Ks, Vs, q, p, maxb, idx, cnt):
             H.check_selection(idx[b, h, :n], scores, n, p.n_local_blocks)
 
 
-def test_select_many_small_units_and_repeat():
+@pytest.mark.parametrize("maxb", [72, 6150])  # one-CTA and cluster top-n
+def test_select_many_small_units_and_repeat(maxb):
     """More (sequence, KV head) units than SMs, of one or two score pieces
     each, ragged lengths and two empty sequences (count 0, ids -1). A second
     call on the same state must give the same result."""
@@ -154,8 +161,7 @@ def test_select_many_small_units_and_repeat():
     lens[3] = 0
     lens[50] = 0
     Ks, Vs = seq_inputs(72, B, Hkv, lens)
-    maxb = 72
-    cache = H.make_cache(Ks, Vs, g * Hkv, maxb)
+    cache = H.make_cache(Ks, Vs, g * Hkv, maxb, compact=True)
     q = synth.normal_bf16(synth.rng(73), (B, g * Hkv, 128))
     p = resa.params(0.2, 2, 1)
     n_cap = resa.resa_max_selected(cache.struct, p)
@@ -181,13 +187,14 @@ def test_select_large_unit():
     check_select_case(cache, Ks, Vs, q, p, maxb, idx, cnt)
 
 
-def test_select_ties_go_to_lower_index():
+@pytest.mark.parametrize("maxb", [44, 6200])  # one-CTA and cluster top-n
+def test_select_ties_go_to_lower_index(maxb):
     """Identical blocks give identical scores; the lower ids must win."""
     Hkv, g, T = 1, 4, 16 * 40
     blk = synth.normal_bf16(synth.rng(6), (Hkv, 16, 128))
     K = np.tile(blk, (1, 40, 1))
     V = synth.normal_bf16(synth.rng(7), (Hkv, T, 128))
-    cache = H.make_cache([K], [V], g, 44)
+    cache = H.make_cache([K], [V], g, maxb, compact=True)
     q = synth.normal_bf16(synth.rng(8), (1, g, 128))
     p = resa.params(0.1, 0, 1)
     idx, cnt = run_select(cache, q, p, 16)
@@ -195,9 +202,10 @@ def test_select_ties_go_to_lower_index():
     assert idx[0, 0, :4].tolist() == [0, 1, 2, 39]
 
 
-def test_select_budget_over_cap_is_reported_and_clamped():
+@pytest.mark.parametrize("maxb", [110, 6200])  # one-CTA and cluster top-n
+def test_select_budget_over_cap_is_reported_and_clamped(maxb):
     Ks, Vs = seq_inputs(9, 1, 1, [1600])
-    cache = H.make_cache(Ks, Vs, 2, 110)
+    cache = H.make_cache(Ks, Vs, 2, maxb, compact=True)
     q = synth.normal_bf16(synth.rng(9), (1, 2, 128))
     p = resa.params(0.1, 0, 1)
     idx, cnt = run_select(cache, q, p, 5)               # n = 10 > n_cap = 5
