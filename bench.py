@@ -271,8 +271,9 @@ class LayerCache:
         self.out = torch.empty((f, B, Hq, HEAD_DIM), dtype=torch.bfloat16, device=device)
         self.rout = torch.empty((B, f, Hq, HEAD_DIM), dtype=torch.bfloat16, device=device)
 
-    # each call below launches: commit 1 kernel, select 2, decode 2, rectify 2
-    KERNELS_PER_DECODE_STEP = 5
+    # kernels per call: the fused decode step 4 (score, top-n, decode, merge),
+    # rectify 2, overwrite 1
+    KERNELS_PER_DECODE_STEP = 4
     KERNELS_PER_RECTIFY = 3
 
     def commit(self, t):
@@ -294,10 +295,10 @@ class LayerCache:
         self.resa.resa_commit_kv(self.cache.struct, self.rk, self.rv, self.w.f, True)
 
     def decode(self, t):
-        """One decode step of Algorithm 1 for this layer (commit, select, decode)."""
-        self.commit(t)
-        self.select(t)
-        self.sparse_decode(t)
+        """One decode step of Algorithm 1 for this layer: the fused call that
+        appends the token, selects and decodes (= commit + select + decode)."""
+        self.resa.resa_decode_step(self.cache.struct, self.k[t], self.v[t], self.q[t], self.p, self.idx, self.cnt,
+                                   self.n_cap, self.out[t], None, 0, self.ws, self.ws_bytes)
 
     def rectify(self):
         """Rectification branch of Algorithm 1 for this layer."""
@@ -406,7 +407,9 @@ def config_of(w: synth.Workload, args) -> dict:
     return {"workload": w.name, "batch": w.batch, "context": w.context, "q_heads": w.num_q_heads,
             "kv_heads": w.num_kv_heads, "head_dim": HEAD_DIM, "block_size": BLOCK, "keep": w.keep,
             "n_min_blocks": w.n_min_blocks, "n_local_blocks": w.n_local_blocks, "f": w.f,
-            "layers_rotated": args.layers, "step": f"{w.f} decode steps + 1 rectification per layer",
+            "layers_rotated": args.layers,
+            "step": f"{w.f} decode steps (resa_decode_step: append + select + decode) + 1 rectification "
+                    f"(resa_rectify_attention + overwrite commit) per layer",
             "l2": f"{args.layers} independent layer caches rotated per decode step (other layers' traffic "
                   f"between reuses exceeds the 129 MB L2)", "parallelism": f"replicas x{args.gpus} (weak)"}
 
@@ -458,7 +461,7 @@ def run_ours(args, w: synth.Workload):
 
     L, f, B = args.layers, w.f, w.batch
     # periods that append f tokens: warm-up call, graph warm-up/timed/e2e replays, attribution commits
-    periods_total = 1 + args.warmup + args.steps + args.steps + 1 + 2 * ATTR_REPS
+    periods_total = 1 + args.warmup + args.steps + args.steps + 2 * (1 + ATTR_REPS)
     capacity = ((w.context + f * periods_total + BLOCK) // BLOCK + 1) * BLOCK
     layers = [LayerCache(w, capacity, w.seed * 100 + 17 * rank + i, device) for i in range(L)]
     torch.cuda.synchronize()
@@ -498,28 +501,38 @@ def run_ours(args, w: synth.Workload):
     T += f * args.steps
 
     # ---- per-call durations: one graph per call type, the period's calls of that type in order ----
+    # The step is decode_step (f x L), rectify and overwrite (L each); select,
+    # decode and commit are the pieces decode_step fuses, timed as their own
+    # calls for the per-kernel rooflines.
     T_attr = T
+    appends = ("decode_step", "commit")
     kinds = {
+        "decode_step": lambda: [Lc.decode(t) for t in range(f) for Lc in layers],
         "select": lambda: [Lc.select(t) for t in range(f) for Lc in layers],
         "decode": lambda: [Lc.sparse_decode(t) for t in range(f) for Lc in layers],
         "rectify": lambda: [Lc.rectify_attention() for Lc in layers],
         "overwrite": lambda: [Lc.overwrite() for Lc in layers],
         "commit": lambda: [Lc.commit(t) for t in range(f) for Lc in layers],
     }
-    ncalls = {"select": f * L, "decode": f * L, "rectify": L, "overwrite": L, "commit": f * L}
+    ncalls = {"decode_step": f * L, "select": f * L, "decode": f * L, "rectify": L, "overwrite": L, "commit": f * L}
+    in_step = ("decode_step", "rectify", "overwrite")
     mean_us = {}
     for kind, fn in kinds.items():
         gk = capture(fn, device)             # capture does not execute
         gk.replay()                          # warm
-        if kind == "commit":
+        if kind in appends:
             T += f
         mean_us[kind] = time_graph(gk, ATTR_REPS) / ncalls[kind] * 1e6
-        if kind == "commit":
+        if kind in appends:
             T += f * ATTR_REPS
         del gk
     check_device_errors(layers)
     Tm = T_attr + f // 2
     algo = {
+        "decode_step": (commit_bytes(B, w.num_kv_heads, 1) +
+                        select_bytes(B, w.num_q_heads, w.num_kv_heads, Tm, w.keep, w.n_min_blocks, w.n_local_blocks) +
+                        decode_bytes(B, w.num_q_heads, w.num_kv_heads, T_attr, w.keep, w.n_min_blocks,
+                                     w.n_local_blocks)),
         "commit": commit_bytes(B, w.num_kv_heads, 1),
         "select": select_bytes(B, w.num_q_heads, w.num_kv_heads, Tm, w.keep, w.n_min_blocks, w.n_local_blocks),
         "decode": decode_bytes(B, w.num_q_heads, w.num_kv_heads, T_attr, w.keep, w.n_min_blocks,
@@ -530,20 +543,27 @@ def run_ours(args, w: synth.Workload):
     peaks, peak_kind = load_peaks()
     hbm = float(peaks["hbm_gbs"])
     per_step_us = {k: mean_us[k] * ncalls[k] for k in mean_us}
-    tot = sum(per_step_us.values())
+    tot = sum(per_step_us[k] for k in in_step)
     calls = {}
     for k in mean_us:
         gbs = algo[k] / (mean_us[k] * 1e-6) / 1e9
         calls[k] = {"us_per_call": round(mean_us[k], 2), "calls_per_step": ncalls[k], "GB/s": round(gbs, 1),
-                    "frac_hbm": round(gbs / hbm, 3), "share_of_step": round(per_step_us[k] / tot, 3),
-                    "algorithmic_bytes": int(algo[k])}
+                    "frac_hbm": round(gbs / hbm, 3), "algorithmic_bytes": int(algo[k])}
+        if k in in_step:
+            calls[k]["share_of_step"] = round(per_step_us[k] / tot, 3)
+        else:
+            calls[k]["part_of"] = "decode_step"
+            calls[k]["share_of_decode_step"] = round(mean_us[k] / mean_us["decode_step"], 3)
     rflops = rectify_flops(B, w.num_q_heads, T_attr, f)
     calls["rectify"]["TFLOP/s"] = round(rflops / (mean_us["rectify"] * 1e-6) / 1e12, 1)
     calls["rectify"]["frac_bf16_sustained"] = round(rflops / (mean_us["rectify"] * 1e-6) / 1e12 /
                                                     float(peaks["bf16_tflops_sustained"]), 3)
-    dominant = max(per_step_us, key=per_step_us.get)
+    # dominant kernel pair: the largest per-step time among the separately
+    # timed calls (select and decode stand for their share of decode_step)
+    dominant = max((k for k in per_step_us if k != "decode_step"), key=per_step_us.get)
+    topn = "topn_cta_kernel" if layers[0].cache.max_blocks <= TOPN_CTA_MAX_BLOCKS else "topn_kernel"
     kernel, src = {"decode": ("sparse_decode_kernel+merge_kernel", "sparse_decode.cu"),
-                   "select": ("score_kernel+topn_kernel", "select.cu"),
+                   "select": ("score_kernel+" + topn, "select.cu"),
                    "rectify": ("rectify_kernel+merge_kernel", "rectify.cu"),
                    "commit": ("commit_append_kernel", "kv_commit.cu"),
                    "overwrite": ("commit_overwrite_kernel", "kv_commit.cu")}[dominant]
@@ -581,6 +601,7 @@ def run_ours(args, w: synth.Workload):
 
 
 ATTR_REPS = 3
+TOPN_CTA_MAX_BLOCKS = 6144  # caches of up to this many blocks per sequence use the one-CTA top-n
 
 
 def run_e2e(args, layers, graph):

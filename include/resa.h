@@ -221,6 +221,25 @@ resa_status_t resa_sparse_decode(const resa_cache_t* cache, const void* q, const
                                  void* stream);
 
 /*
+ * One sparse decode step of Algorithm 1 in one call: the append commit of one
+ * token (k_new, v_new; bf16 [batch][num_kv_heads][head_dim]), block
+ * selection (Eq. 4, Eq. 5) and block-sparse decoding (Eq. 2, Algorithm 2) --
+ * the same results, bit for bit, as resa_commit_kv(n_tokens = 1, append)
+ * followed by resa_select_blocks and resa_sparse_decode on the same arguments,
+ * without the commit's own launch: the scoring pass writes the new key and
+ * value into their page and folds the key into its block's summary before it
+ * scores that block, and the combine kernel advances seq_lens[b] by one at the
+ * end. Arguments are those of the three calls; the workspace must hold both
+ * the scores and the split partials (resa_workspace_size covers it).
+ * Device errors: as in the three calls; a sequence already at capacity is
+ * reported (RESA_DEV_SEQ_LEN_RANGE), gets count 0, and keeps its length.
+ */
+resa_status_t resa_decode_step(const resa_cache_t* cache, const void* k_new, const void* v_new, const void* q,
+                               const resa_params_t* params, int32_t* indices, int32_t* counts, int32_t n_cap,
+                               void* out, float* lse, int32_t num_splits, void* workspace, size_t workspace_bytes,
+                               void* stream);
+
+/*
  * Dense rectification attention (Section 2.2; Algorithm 1 DenseForward):
  * the f most recent tokens of each sequence, at positions
  * [seq_lens[b] - f, seq_lens[b]), attend causally to the whole cache: query

@@ -16,36 +16,6 @@
 namespace resa {
 namespace {
 
-__device__ __forceinline__ void minmax8(const uint4& v, float* mn, float* mx) {
-  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const float lo = bf16_lo(w[i]), hi = bf16_hi(w[i]);
-    mn[2 * i] = fminf(mn[2 * i], lo);
-    mx[2 * i] = fmaxf(mx[2 * i], lo);
-    mn[2 * i + 1] = fminf(mn[2 * i + 1], hi);
-    mx[2 * i + 1] = fmaxf(mx[2 * i + 1], hi);
-  }
-}
-
-// min/max of bf16 inputs are bf16 values: dropping the low 16 bits is exact.
-__device__ __forceinline__ uint4 to_bf16x8(const float* x) {
-  uint4 r;
-  r.x = (__float_as_uint(x[0]) >> 16) | (__float_as_uint(x[1]) & 0xFFFF0000u);
-  r.y = (__float_as_uint(x[2]) >> 16) | (__float_as_uint(x[3]) & 0xFFFF0000u);
-  r.z = (__float_as_uint(x[4]) >> 16) | (__float_as_uint(x[5]) & 0xFFFF0000u);
-  r.w = (__float_as_uint(x[6]) >> 16) | (__float_as_uint(x[7]) & 0xFFFF0000u);
-  return r;
-}
-
-__device__ __forceinline__ size_t pool_off(const CacheView& c, int page, int h, int row) {
-  return ((static_cast<size_t>(page) * c.Hkv + h) * kBlock + row) * kHeadDim;
-}
-
-__device__ __forceinline__ size_t summ_off(const CacheView& c, int b, int h, int blk) {
-  return ((static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks + blk) * 2 * kHeadDim;
-}
-
 __global__ void __launch_bounds__(256) commit_append_kernel(CacheView c, const uint16_t* __restrict__ k_new,
                                                             const uint16_t* __restrict__ v_new, int n) {
   pdl_launch_dependents();

@@ -142,6 +142,9 @@ CacheView view(const resa_cache_t* c) {
   v.summ = static_cast<uint16_t*>(c->summaries);
   v.status = c->device_status;
   v.active = nullptr;
+  v.pending = 0;
+  v.k_append = nullptr;
+  v.v_append = nullptr;
   return v;
 }
 
@@ -348,6 +351,50 @@ resa_status_t resa_sparse_decode(const resa_cache_t* cache, const void* q, const
                                        scale_of(cache, params), splits, o_part, lse_part, st);
   if (e == cudaSuccess)
     e = launch_merge(o_part, lse_part, static_cast<int>(rows), splits, static_cast<uint16_t*>(out), lse, st);
+  return e == cudaSuccess ? RESA_OK : RESA_ERR_CUDA;
+}
+
+resa_status_t resa_decode_step(const resa_cache_t* cache, const void* k_new, const void* v_new, const void* q,
+                               const resa_params_t* params, int32_t* indices, int32_t* counts, int32_t n_cap,
+                               void* out, float* lse, int32_t num_splits, void* workspace, size_t workspace_bytes,
+                               void* stream) {
+  resa_status_t s = check_cache(cache);
+  if (s != RESA_OK) return s;
+  if ((s = check_params(params)) != RESA_OK) return s;
+  if (k_new == nullptr || v_new == nullptr || q == nullptr || indices == nullptr || counts == nullptr ||
+      out == nullptr || n_cap <= 0 || num_splits < 0)
+    return RESA_ERR_INVALID_ARG;
+  if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(q)) return RESA_ERR_INVALID_ARG;
+  int splits = num_splits;
+  if (splits == 0 && (s = auto_decode_splits(cache, n_cap, &splits)) != RESA_OK) return s;
+  if (splits > 1024) return RESA_ERR_INVALID_ARG;
+  const size_t rows = static_cast<size_t>(cache->batch) * cache->num_q_heads;
+  if (workspace == nullptr || workspace_bytes < scores_bytes(cache) ||
+      workspace_bytes < partial_bytes(rows, splits))
+    return RESA_ERR_WORKSPACE;
+  int sms = 0;
+  if ((s = sm_count(&sms)) != RESA_OK) return s;
+  CUtensorMap tk, tv;
+  if ((s = pool_tensor_map(cache, cache->k_pool, &tk)) != RESA_OK) return s;
+  if ((s = pool_tensor_map(cache, cache->v_pool, &tv)) != RESA_OK) return s;
+  CacheView v = view(cache);
+  v.pending = 1;
+  v.k_append = static_cast<const uint16_t*>(k_new);
+  v.v_append = static_cast<const uint16_t*>(v_new);
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // scores and partials alias: the partials are written after the top-n has read the scores
+  cudaError_t e = launch_select(v, static_cast<const uint16_t*>(q), params->keep_ratio, params->n_min_blocks,
+                                params->n_local_blocks, indices, counts, n_cap, static_cast<float*>(workspace), sms,
+                                st);
+  float* o_part = static_cast<float*>(workspace);
+  float* lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) +
+                                             align_up(rows * splits * kHeadDimHost * sizeof(float)));
+  if (e == cudaSuccess)
+    e = launch_sparse_decode(v, tk, tv, static_cast<const uint16_t*>(q), indices, counts, n_cap,
+                             scale_of(cache, params), splits, o_part, lse_part, st);
+  if (e == cudaSuccess)
+    e = launch_merge(o_part, lse_part, static_cast<int>(rows), splits, static_cast<uint16_t*>(out), lse, st, nullptr,
+                     cache->num_q_heads, &v);
   return e == cudaSuccess ? RESA_OK : RESA_ERR_CUDA;
 }
 

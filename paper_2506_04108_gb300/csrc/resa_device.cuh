@@ -26,6 +26,29 @@ __device__ __forceinline__ void record_error(int32_t* status, int32_t code, int3
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
+// Folds 8 bf16 values (one 16-byte piece) into running fp32 min/max (Eq. 3).
+__device__ __forceinline__ void minmax8(const uint4& v, float* mn, float* mx) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float lo = bf16_lo(w[i]), hi = bf16_hi(w[i]);
+    mn[2 * i] = fminf(mn[2 * i], lo);
+    mx[2 * i] = fmaxf(mx[2 * i], lo);
+    mn[2 * i + 1] = fminf(mn[2 * i + 1], hi);
+    mx[2 * i + 1] = fmaxf(mx[2 * i + 1], hi);
+  }
+}
+
+// min/max of bf16 inputs are bf16 values: dropping the low 16 bits is exact.
+__device__ __forceinline__ uint4 to_bf16x8(const float* x) {
+  uint4 r;
+  r.x = (__float_as_uint(x[0]) >> 16) | (__float_as_uint(x[1]) & 0xFFFF0000u);
+  r.y = (__float_as_uint(x[2]) >> 16) | (__float_as_uint(x[3]) & 0xFFFF0000u);
+  r.z = (__float_as_uint(x[4]) >> 16) | (__float_as_uint(x[5]) & 0xFFFF0000u);
+  r.w = (__float_as_uint(x[6]) >> 16) | (__float_as_uint(x[7]) & 0xFFFF0000u);
+  return r;
+}
+
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);

@@ -26,7 +26,24 @@ struct CacheView {
   uint16_t* summ;
   int32_t* status;
   const int32_t* active;  // [B]: sequences with 0 are left out of commits and rectification; null = all
+  // Fused decode step: `pending` tokens (0 or 1) are appended by the running
+  // call and not yet counted in seq_lens, which its last kernel advances;
+  // every kernel of the call works on T = seq_lens[b] + pending. The appended
+  // key and value are k_append / v_append, bf16 [B][Hkv][128].
+  int pending;
+  const uint16_t* k_append;
+  const uint16_t* v_append;
 };
+
+#ifdef __CUDACC__
+// Element offsets into the paged pool and the block summaries.
+__device__ __forceinline__ size_t pool_off(const CacheView& c, int page, int h, int row) {
+  return ((static_cast<size_t>(page) * c.Hkv + h) * 16 + row) * 128;
+}
+__device__ __forceinline__ size_t summ_off(const CacheView& c, int b, int h, int blk) {
+  return ((static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks + blk) * 2 * 128;
+}
+#endif
 
 // Launches `kernel` with programmatic stream serialization (see
 // pdl_launch_dependents / pdl_wait in resa_device.cuh).
@@ -67,8 +84,11 @@ int decode_ctas_per_sm();  // resident decode CTAs per SM (occupancy), >= 1
 cudaError_t launch_sparse_decode(const CacheView& c, const CUtensorMap& tm_k, const CUtensorMap& tm_v,
                                  const uint16_t* q, const int32_t* indices, const int32_t* counts, int n_cap,
                                  float sm_scale, int splits, float* o_part, float* lse_part, cudaStream_t st);
+// `advance` (a fused decode step's view, pending > 0): the merge also counts
+// the appended token in seq_lens; rows_per_seq must then be Hq.
 cudaError_t launch_merge(const float* o_part, const float* lse_part, int rows, int splits, uint16_t* out,
-                         float* lse_out, cudaStream_t st, const int32_t* active = nullptr, int rows_per_seq = 1);
+                         float* lse_out, cudaStream_t st, const int32_t* active = nullptr, int rows_per_seq = 1,
+                         const CacheView* advance = nullptr);
 
 // rectify.cu
 int rectify_row_groups(int g, int f);

@@ -90,6 +90,7 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c,
   extern __shared__ __align__(1024) uint8_t smem[];
   // per-sequence block counts and the piece prefix over (sequence, head) units
   __shared__ int sh_M[kMaxBatch];
+  __shared__ int sh_T[kMaxBatch];
   __shared__ int sh_pref[kMaxBatch + 1];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   uint8_t* ring = smem + warp * kScoreStages * kPieceBytes;
@@ -103,8 +104,10 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c,
   // over sequences (lengths out of range count as empty: top-n reports them)
   auto build_tables = [&]() {
     for (int b = tid; b < c.B; b += blockDim.x) {
-      const int T = c.seq_lens[b];
-      sh_M[b] = (T < 0 || T > c.max_blocks * kBlock) ? 0 : (T + kBlock - 1) / kBlock;
+      const int T = c.seq_lens[b] + c.pending;
+      const bool bad = T < 0 || T > c.max_blocks * kBlock;
+      sh_M[b] = bad ? 0 : (T + kBlock - 1) / kBlock;
+      sh_T[b] = bad ? 0 : T;
     }
     __syncthreads();
     if (warp == 0) {
@@ -189,6 +192,7 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c,
   int cur_unit = -1, k_fail = -1;
   float qa[8];
   uint32_t sg[4];
+  uint4 ka = make_uint4(0, 0, 0, 0), va = ka;  // the appended token's key / value, this lane's 8 dims
   for (int k = 0; k < nmine; ++k) {
     const int st = k % kScoreStages;
     int b, h, blk0, nblk;
@@ -196,6 +200,11 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c,
     const int unit = b * c.Hkv + h;
     if (unit != cur_unit) {  // pooled query (mean of the group's heads), this lane's 8 dims
       cur_unit = unit;
+      if (c.pending) {
+        const size_t kv = (static_cast<size_t>(b) * c.Hkv + h) * kHeadDim + ch * 8;
+        ka = *reinterpret_cast<const uint4*>(c.k_append + kv);
+        va = *reinterpret_cast<const uint4*>(c.v_append + kv);
+      }
       float qp[8];
 #pragma unroll
       for (int j = 0; j < 8; ++j) qp[j] = 0.f;
@@ -231,7 +240,46 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c,
       break;
     }
     mbar_try_wait(bar0 + 8 * st, (k / kScoreStages) & 1);
-    const uint8_t* piece = ring + st * kPieceBytes;
+    uint8_t* piece = ring + st * kPieceBytes;
+    if (c.pending) {
+      // Fused decode step: the appended token lands in block (T - 1) / 16.
+      // The warp holding that block folds the key into its summary (Eq. 3,
+      // online; a block the token opens starts empty), scores the updated
+      // summary, and writes it, the key and the value to the cache.
+      const int T = sh_T[b], last = (T - 1) >> 4;
+      if (last >= blk0 && last < blk0 + nblk) {
+        if (half == 0) {
+          uint8_t* ps = piece + (last - blk0) * 512;
+          float mn[8], mx[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            mn[j] = __int_as_float(0x7f800000);
+            mx[j] = -__int_as_float(0x7f800000);
+          }
+          if (((T - 1) & (kBlock - 1)) != 0) {
+            minmax8(*reinterpret_cast<const uint4*>(ps + ch * 16), mn, mx);
+            minmax8(*reinterpret_cast<const uint4*>(ps + 256 + ch * 16), mn, mx);
+          }
+          minmax8(ka, mn, mx);
+          const uint4 smin = to_bf16x8(mn), smax = to_bf16x8(mx);
+          *reinterpret_cast<uint4*>(ps + ch * 16) = smin;
+          *reinterpret_cast<uint4*>(ps + 256 + ch * 16) = smax;
+          fence_proxy_async_smem();  // the stage is refilled by a bulk copy later
+          uint16_t* sd = c.summ + summ_off(c, b, h, last);
+          *reinterpret_cast<uint4*>(sd + ch * 8) = smin;
+          *reinterpret_cast<uint4*>(sd + kHeadDim + ch * 8) = smax;
+          const int page = c.page_table[static_cast<size_t>(b) * c.max_blocks + last];
+          if (page < 0 || page >= c.num_pages) {
+            if (ch == 0) record_error(c.status, RESA_DEV_PAGE_RANGE, b);
+          } else {
+            const size_t dst = pool_off(c, page, h, (T - 1) & (kBlock - 1)) + ch * 8;
+            *reinterpret_cast<uint4*>(c.k_pool + dst) = ka;
+            *reinterpret_cast<uint4*>(c.v_pool + dst) = va;
+          }
+        }
+        __syncwarp();
+      }
+    }
     float* out = scores + static_cast<size_t>(unit) * c.max_blocks + blk0;
 #pragma unroll
     for (int v = 0; v < kPieceBlocks / 2; ++v) {
@@ -337,7 +385,7 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
   const int b = blockIdx.z, h = blockIdx.y;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   int32_t* out = indices + (static_cast<size_t>(b) * c.Hkv + h) * n_cap;
-  const int T = __ldcg(c.seq_lens + b);  // final before the score kernel let this one launch
+  const int T = __ldcg(c.seq_lens + b) + c.pending;  // final before the score kernel let this one launch
   pdl_wait();                            // the scores
   if (T < 0 || T > c.max_blocks * kBlock) {  // the whole cluster takes this branch
     if (rank == 0 && tid == 0) {
@@ -581,7 +629,7 @@ __global__ void __launch_bounds__(kTopnCtaThreads, 1) topn_cta_kernel(CacheView 
   pdl_launch_dependents();
   const int h = blockIdx.x, b = blockIdx.y;
   int32_t* out = indices + (static_cast<size_t>(b) * c.Hkv + h) * n_cap;
-  const int T = __ldcg(c.seq_lens + b);  // final before the score kernel let this one launch
+  const int T = __ldcg(c.seq_lens + b) + c.pending;  // final before the score kernel let this one launch
   if (T < 0 || T > c.max_blocks * kBlock) {
     pdl_wait();
     if (tid == 0) {

@@ -74,7 +74,7 @@ __global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid
   const int nj_cap = max(0, min(a.n_cap, j0 + per) - j0);
   const int cnt_cap = nj_cap > warp ? (nj_cap - warp + kWarps - 1) / kWarps : 0;
   const int32_t* idx = a.indices + static_cast<size_t>(b * c.Hkv + h) * a.n_cap + j0 + warp;
-  const int T = c.seq_lens[b];
+  const int T = c.seq_lens[b] + c.pending;
   int n = a.counts[b * c.Hkv + h];
   int pre_blk = lane < cnt_cap ? idx[lane * kWarps] : -1;
   if (T < 0 || T > c.max_blocks * kBlock) {
@@ -290,6 +290,15 @@ __global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid
   }
 }
 
+// Length advance of a fused decode step: the merge is its last kernel, so it
+// counts the appended token in seq_lens (row 0 of each sequence; a length
+// that the call found out of range is left as it is).
+struct LenAdvance {
+  int32_t* lens;  // null: no advance
+  int pending;
+  int cap;        // max_blocks * 16
+};
+
 // One CTA of 8 warps per output row. Warp w takes the splits w, w + 8, ...:
 // its lanes load ten partial rows (16 bytes each) and their log2-sum-exps at
 // once, so up to 80 splits cost one round of loads; each warp keeps its sum
@@ -303,12 +312,17 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const float* __
                                                                  uint16_t* __restrict__ out,
                                                                  float* __restrict__ lse_out,
                                                                  const int32_t* __restrict__ active,
-                                                                 int rows_per_seq) {
+                                                                 int rows_per_seq, LenAdvance adv) {
   __shared__ float4 red[kMergeWarps][kHeadDim / 4];
   __shared__ float wmax[kMergeWarps];
   pdl_launch_dependents();
   pdl_wait();
   const size_t row = blockIdx.x;
+  if (adv.lens != nullptr && threadIdx.x == 0 && row % rows_per_seq == 0) {
+    const int b = static_cast<int>(row / rows_per_seq);
+    const int T = adv.lens[b];
+    if (T >= 0 && T + adv.pending <= adv.cap) adv.lens[b] = T + adv.pending;
+  }
   if (active != nullptr && active[row / rows_per_seq] == 0) return;  // a sequence left out of the call
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const float* lp = lse_part + row * splits;
@@ -405,10 +419,14 @@ cudaError_t launch_sparse_decode(const CacheView& c, const CUtensorMap& tm_k, co
 }
 
 cudaError_t launch_merge(const float* o_part, const float* lse_part, int rows, int splits, uint16_t* out,
-                         float* lse_out, cudaStream_t st, const int32_t* active, int rows_per_seq) {
+                         float* lse_out, cudaStream_t st, const int32_t* active, int rows_per_seq,
+                         const CacheView* advance) {
   if (rows == 0) return cudaSuccess;
+  LenAdvance adv{nullptr, 0, 0};
+  if (advance != nullptr && advance->pending > 0)
+    adv = LenAdvance{advance->seq_lens, advance->pending, advance->max_blocks * kBlock};
   return launch_pdl(merge_kernel, dim3(rows), dim3(kMergeWarps * 32), 0, st, o_part, lse_part, splits, out,
-                    lse_out, active, rows_per_seq);
+                    lse_out, active, rows_per_seq, adv);
 }
 
 }  // namespace resa

@@ -27,7 +27,7 @@ DEVICE_ERRORS = {0: "RESA_DEV_OK", 1: "RESA_DEV_SEQ_LEN_RANGE", 2: "RESA_DEV_PAG
 EXPORTED = ["resa_abi_version", "resa_status_string", "resa_max_selected", "resa_decode_num_splits",
             "resa_workspace_size", "resa_update_summaries", "resa_commit_kv", "resa_select_blocks",
             "resa_sparse_decode", "resa_rectify_attention", "resa_read_device_error", "resa_sparse_decode_static",
-            "resa_commit_kv_active", "resa_rectify_attention_active"]
+            "resa_commit_kv_active", "resa_rectify_attention_active", "resa_decode_step"]
 
 
 class ResaError(RuntimeError):
@@ -76,6 +76,7 @@ def load() -> ctypes.CDLL:
         "resa_sparse_decode_static": ([cp, pp, pp, pp, c_int32, pc, pp, pp, c_int32, pp], c_int32),
         "resa_commit_kv_active": ([cp, pp, pp, pp, c_int32, c_int32, pp], c_int32),
         "resa_rectify_attention_active": ([cp, pp, pp, pp, pp, c_int32, pc, pp, pp, pp, c_size_t, pp], c_int32),
+        "resa_decode_step": ([cp, pp, pp, pp, pc, pp, pp, c_int32, pp, pp, c_int32, pp, c_size_t, pp], c_int32),
     }
     for name, (args, ret) in sig.items():
         fn = getattr(L, name)
@@ -159,6 +160,15 @@ def resa_sparse_decode(cache: ResaCacheT, q, indices, counts, n_cap: int, p: Res
     _check(load().resa_sparse_decode(ctypes.byref(cache), _ptr(q), _ptr(indices), _ptr(counts), n_cap,
                                      ctypes.byref(p), _ptr(out), _ptr(lse), num_splits, _ptr(workspace),
                                      workspace_bytes, _stream(stream)), "resa_sparse_decode")
+
+
+def resa_decode_step(cache: ResaCacheT, k_new, v_new, q, p: ResaParamsT, indices, counts, n_cap: int, out, lse,
+                     num_splits: int, workspace, workspace_bytes: int, stream=None):
+    """One decode step in one call: append (k_new, v_new), select, decode;
+    equal to resa_commit_kv + resa_select_blocks + resa_sparse_decode."""
+    _check(load().resa_decode_step(ctypes.byref(cache), _ptr(k_new), _ptr(v_new), _ptr(q), ctypes.byref(p),
+                                   _ptr(indices), _ptr(counts), n_cap, _ptr(out), _ptr(lse), num_splits,
+                                   _ptr(workspace), workspace_bytes, _stream(stream)), "resa_decode_step")
 
 
 def resa_sparse_decode_static(cache: ResaCacheT, q, indices, counts, n_cap: int, p: ResaParamsT, out, lse,

@@ -27,16 +27,17 @@ def host_f64(t: torch.Tensor) -> np.ndarray:
     return O.widen_bf16(host_bits(t))
 
 
-def make_cache(Ks, Vs, Hq, max_blocks, seed=1, zero_pools=False, compact=False):
+def make_cache(Ks, Vs, Hq, max_blocks, seed=1, zero_pools=False, compact=False, reserve_blocks=0):
     """Paged cache holding per-sequence keys/values Ks[b], Vs[b] (uint16 bits,
     [Hkv, T_b, d]; ragged T_b allowed), pages scattered by a seeded page table.
     Summaries are built with resa_update_summaries. `compact` gives pages only
-    to the blocks the sequences hold (the rest of each page-table row points at
-    page 0): for wide page-table rows whose tail is never touched."""
+    to the blocks the sequences hold plus `reserve_blocks` more each (the rest
+    of each page-table row points at page 0): for wide page-table rows whose
+    tail is never touched."""
     B = len(Ks)
     Hkv = Ks[0].shape[0]
     if compact:
-        need = [(K.shape[1] + 15) // 16 for K in Ks]
+        need = [min(max_blocks, (K.shape[1] + 15) // 16 + reserve_blocks) for K in Ks]
         perm = synth.rng(seed).permutation(max(1, sum(need))).astype(np.int32)
         pt = np.zeros((B, max_blocks), dtype=np.int32)
         off = 0

@@ -98,6 +98,13 @@ def test_bad_call_arguments_rejected_on_host(lib):
                                       1 << 20, None) == 1
     assert lib.resa_rectify_attention(cp, 0x70000, 0, 0x72000, 8, ctypes.byref(P), 0x4000, None, 0x3000,
                                       1 << 20, None) == 1
+    # fused decode step: argument checks precede any CUDA call (explicit splits)
+    def step(k=0x70000, v=0x71000, q=0x72000, n_cap=10, out=0x4000, splits=4, ws=0x3000, wsb=1 << 20):
+        return lib.resa_decode_step(cp, k, v, q, ctypes.byref(P), 0x1000, 0x2000, n_cap, out, None, splits, ws, wsb,
+                                    None)
+    assert step(k=0) == 1 and step(v=0) == 1 and step(q=0) == 1 and step(out=0) == 1
+    assert step(v=0x71008) == 1 and step(n_cap=0) == 1 and step(splits=-1) == 1 and step(splits=2000) == 1
+    assert step(wsb=16) == 3 and step(ws=0) == 3
 
 
 @pytest.mark.parametrize("max_blocks,keep,n_min,n_local", [(256, 0.1, 16, 4), (2048, 0.1, 128, 1),

@@ -1,7 +1,7 @@
 """Algorithm 1 end to end through the C ABI against the fp64 oracle.
 
 Each decode step: commit the step's (sparse-era) K/V -> select blocks ->
-sparse decode; every f steps: rectification attention over the dense
+sparse decode (three calls, or the one fused resa_decode_step); every f steps: rectification attention over the dense
 q/k/v of the last f tokens, then the overwrite commit. Selections are
 compared per (sequence, KV head) with the near-tie rule and outputs with
 2e-2 max-abs / 1e-3 mean-abs (against the oracle recomputed on the GPU's
@@ -24,8 +24,8 @@ pytestmark = pytest.mark.gpu
 class GpuLoop:
     """The decode path of Algorithm 1 driven through the C ABI."""
 
-    def __init__(self, w: synth.Workload, inp: synth.HostDecodeInputs, steps: int):
-        self.w, self.inp = w, inp
+    def __init__(self, w: synth.Workload, inp: synth.HostDecodeInputs, steps: int, fused: bool = False):
+        self.w, self.inp, self.fused = w, inp, fused
         B, Hkv = inp.prefill_k.shape[:2]
         self.B, self.Hkv, self.Hq = B, Hkv, w.num_q_heads
         T0 = inp.prefill_k.shape[2]
@@ -45,11 +45,15 @@ class GpuLoop:
         c = self.cache.struct
         k = H.dev_bf16(self.inp.step_k[i][:, None])       # [B, 1, Hkv, d]
         v = H.dev_bf16(self.inp.step_v[i][:, None])
-        resa.resa_commit_kv(c, k, v, 1, False)
         q = H.dev_bf16(self.inp.step_q[i])
-        resa.resa_select_blocks(c, q, self.p, self.idx, self.cnt, self.n_cap, self.ws, self.wsb)
-        resa.resa_sparse_decode(c, q, self.idx, self.cnt, self.n_cap, self.p, self.out, self.lse, 0, self.ws,
-                                self.wsb)
+        if self.fused:
+            resa.resa_decode_step(c, k, v, q, self.p, self.idx, self.cnt, self.n_cap, self.out, self.lse, 0,
+                                  self.ws, self.wsb)
+        else:
+            resa.resa_commit_kv(c, k, v, 1, False)
+            resa.resa_select_blocks(c, q, self.p, self.idx, self.cnt, self.n_cap, self.ws, self.wsb)
+            resa.resa_sparse_decode(c, q, self.idx, self.cnt, self.n_cap, self.p, self.out, self.lse, 0, self.ws,
+                                    self.wsb)
         return self.idx.cpu().numpy(), self.cnt.cpu().numpy(), H.host_f64(self.out)
 
     def rectify(self, i):
@@ -63,8 +67,8 @@ class GpuLoop:
         return H.host_f64(self.rout)
 
 
-def run_and_compare(w: synth.Workload, inp: synth.HostDecodeInputs, steps: int, check_seqs):
-    gl = GpuLoop(w, inp, steps)
+def run_and_compare(w: synth.Workload, inp: synth.HostDecodeInputs, steps: int, check_seqs, fused=False):
+    gl = GpuLoop(w, inp, steps, fused)
     g = w.group
     p = O.ResaParams(w.keep, w.n_min_blocks, w.n_local_blocks)
     sc = 1 / math.sqrt(128)
@@ -114,21 +118,24 @@ def test_loop_b1_h8kv2_ctx4k_f8_full():
     assert exact + near == w.steps * w.num_kv_heads
 
 
-def test_loop_qwen_shape_reduced_context():
+@pytest.mark.parametrize("fused", [False, True])
+def test_loop_qwen_shape_reduced_context(fused):
     """Qwen2.5-7B head geometry with K channel outliers, 2 sequences at 3000
     tokens (ragged tail), 40 steps with f = 32 (one rectification)."""
     w = synth.WORKLOADS["qwen7b_b8_ctx32k_f32"]
     inp = synth.decode_inputs(w, context=3000, steps=40, batch=2)
-    run_and_compare(w, inp, 40, [0, 1])
+    run_and_compare(w, inp, 40, [0, 1], fused)
 
 
+@pytest.mark.parametrize("fused", [True, False])
 @pytest.mark.parametrize("name,sample", [("qwen7b_b8_ctx32k_f32", [0, 7]), ("qwen7b_b1_ctx256k_keep5", [0])])
-def test_loop_full_size_sampled(name, sample):
+def test_loop_full_size_sampled(name, sample, fused):
     """Full-size cache and batch, one rectification period; the oracle checks
-    the sampled sequences every step (all KV heads)."""
+    the sampled sequences every step (all KV heads). The fused decode step is
+    the call bench.py times."""
     w = synth.WORKLOADS[name]
     inp = synth.decode_inputs(w, steps=w.f)
-    run_and_compare(w, inp, w.f, sample)
+    run_and_compare(w, inp, w.f, sample, fused)
 
 
 def test_loop_needle_workload_one_layer_sampled():

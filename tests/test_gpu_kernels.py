@@ -214,6 +214,90 @@ def test_select_budget_over_cap_is_reported_and_clamped(maxb):
     assert len(set(idx[0, 0].tolist())) == 5
 
 
+# ------------------------------------------ fused decode step (Alg. 1) ----
+def _decode_step_caches(lens, Hkv, g, maxb, reserve, seed):
+    Ks, Vs = seq_inputs(seed, len(lens), Hkv, lens)
+    mk = lambda: H.make_cache(Ks, Vs, g * Hkv, maxb, zero_pools=True, compact=True, reserve_blocks=reserve)
+    return mk(), mk()
+
+
+@pytest.mark.parametrize("wide", [False, True])  # one-CTA / cluster top-n
+def test_decode_step_equals_commit_select_decode(wide):
+    """resa_decode_step gives, bit for bit, what resa_commit_kv(append 1) +
+    resa_select_blocks + resa_sparse_decode give: ids, counts, outputs and
+    log-sum-exps every step, and the same pools, summaries and lengths after.
+    The ragged lengths put the appended token at every offset of its block
+    over 20 steps (T % 16 = 15 fills a block, 0 opens one); one sequence
+    starts empty."""
+    B, Hkv, g, steps = 4, 2, 4, 20
+    lens = [31, 0, 500, 1000]
+    maxb = 6200 if wide else (max(lens) + steps + 15) // 16 + 2
+    A, F = _decode_step_caches(lens, Hkv, g, maxb, (steps + 15) // 16 + 1, 91)
+    p = resa.params(0.2, 2, 1)
+    n_cap = resa.resa_max_selected(A.struct, p)
+    wa, nb = H.workspace(A, n_cap)
+    wf, _ = H.workspace(F, n_cap)
+    mk = lambda shape, dt: torch.empty(shape, dtype=dt, device="cuda")
+    ia, ifu = mk((B, Hkv, n_cap), torch.int32), mk((B, Hkv, n_cap), torch.int32)
+    ca, cf = mk((B, Hkv), torch.int32), mk((B, Hkv), torch.int32)
+    oa, of = mk((B, g * Hkv, 128), torch.bfloat16), mk((B, g * Hkv, 128), torch.bfloat16)
+    la, lf = mk((B, g * Hkv), torch.float32), mk((B, g * Hkv), torch.float32)
+    gen = synth.rng(92)
+    for t in range(steps):
+        k = H.dev_bf16(synth.normal_bf16(gen, (B, 1, Hkv, 128)))
+        v = H.dev_bf16(synth.normal_bf16(gen, (B, 1, Hkv, 128)))
+        q = H.dev_bf16(synth.normal_bf16(gen, (B, g * Hkv, 128)))
+        resa.resa_commit_kv(A.struct, k, v, 1, False)
+        resa.resa_select_blocks(A.struct, q, p, ia, ca, n_cap, wa, nb)
+        resa.resa_sparse_decode(A.struct, q, ia, ca, n_cap, p, oa, la, 0, wa, nb)
+        resa.resa_decode_step(F.struct, k, v, q, p, ifu, cf, n_cap, of, lf, 0, wf, nb)
+        assert torch.equal(ia, ifu) and torch.equal(ca, cf), t
+        assert np.array_equal(H.host_bits(oa), H.host_bits(of)), t
+        assert np.array_equal(la.cpu().numpy().view(np.uint32), lf.cpu().numpy().view(np.uint32)), t
+    assert resa.resa_read_device_error(A.struct) == (0, 0)
+    assert resa.resa_read_device_error(F.struct) == (0, 0)
+    assert torch.equal(A.seq_lens, F.seq_lens)
+    assert A.seq_lens.cpu().tolist() == [T + steps for T in lens]
+    assert np.array_equal(H.host_bits(A.k_pool), H.host_bits(F.k_pool))
+    assert np.array_equal(H.host_bits(A.v_pool), H.host_bits(F.v_pool))
+    sa, sf = H.host_bits(A.summaries), H.host_bits(F.summaries)
+    for b, T in enumerate(lens):
+        M = (T + steps + 15) // 16
+        assert np.array_equal(sa[b, :, :M], sf[b, :, :M]), b
+
+
+def test_decode_step_sequence_at_capacity():
+    """A sequence whose cache is full cannot take the appended token: the
+    fused step reports RESA_DEV_SEQ_LEN_RANGE, gives it count 0 and ids -1,
+    keeps its length, and serves the other sequences as the three calls do."""
+    Hkv, g, maxb = 1, 4, 20
+    lens = [300, maxb * 16]
+    A, F = _decode_step_caches(lens, Hkv, g, maxb, 2, 93)
+    p = resa.params(0.2, 2, 1)
+    n_cap = resa.resa_max_selected(A.struct, p)
+    wa, nb = H.workspace(A, n_cap)
+    wf, _ = H.workspace(F, n_cap)
+    gen = synth.rng(94)
+    k = H.dev_bf16(synth.normal_bf16(gen, (2, 1, Hkv, 128)))
+    v = H.dev_bf16(synth.normal_bf16(gen, (2, 1, Hkv, 128)))
+    q = H.dev_bf16(synth.normal_bf16(gen, (2, g * Hkv, 128)))
+    mk = lambda shape, dt: torch.empty(shape, dtype=dt, device="cuda")
+    ia, ifu = mk((2, Hkv, n_cap), torch.int32), mk((2, Hkv, n_cap), torch.int32)
+    ca, cf = mk((2, Hkv), torch.int32), mk((2, Hkv), torch.int32)
+    oa, of = mk((2, g * Hkv, 128), torch.bfloat16), mk((2, g * Hkv, 128), torch.bfloat16)
+    resa.resa_commit_kv(A.struct, k, v, 1, False)
+    assert resa.resa_read_device_error(A.struct)[0] == 1
+    resa.resa_select_blocks(A.struct, q, p, ia, ca, n_cap, wa, nb)
+    resa.resa_sparse_decode(A.struct, q, ia, ca, n_cap, p, oa, None, 0, wa, nb)
+    resa.resa_decode_step(F.struct, k, v, q, p, ifu, cf, n_cap, of, None, 0, wf, nb)
+    code, detail = resa.resa_read_device_error(F.struct)
+    assert (code, detail) == (1, 1)
+    assert F.seq_lens.cpu().tolist() == [301, maxb * 16]
+    assert cf[1].cpu().tolist() == [0] and np.all(ifu[1].cpu().numpy() == -1)
+    assert torch.equal(ia[0], ifu[0]) and torch.equal(ca[0], cf[0])
+    assert np.array_equal(H.host_bits(oa[0]), H.host_bits(of[0]))
+
+
 # ------------------------------------------------------ Eq. 2 / Alg. 2 ----
 def run_decode(cache, q_bits, sel_rows, n_cap, p, splits):
     """sel_rows[b][h] = block ids (any order)."""
