@@ -18,8 +18,7 @@ namespace {
 
 __global__ void __launch_bounds__(256) commit_append_kernel(CacheView c, const uint16_t* __restrict__ k_new,
                                                             const uint16_t* __restrict__ v_new, int n) {
-  pdl_launch_dependents();
-  pdl_wait();
+  pdl_wait();  // no early launch of dependents: they may read the summaries and lengths written here
   const int b = blockIdx.x;
   if (c.active != nullptr && c.active[b] == 0) return;
   const int T = c.seq_lens[b];
@@ -74,8 +73,7 @@ __global__ void __launch_bounds__(256) commit_append_kernel(CacheView c, const u
 
 __global__ void __launch_bounds__(256) commit_overwrite_kernel(CacheView c, const uint16_t* __restrict__ k_new,
                                                                const uint16_t* __restrict__ v_new, int n) {
-  pdl_launch_dependents();
-  pdl_wait();
+  pdl_wait();  // no early launch of dependents: they may read the summaries and lengths written here
   const int b = blockIdx.y;
   if (c.active != nullptr && c.active[b] == 0) return;
   const int T = c.seq_lens[b];
@@ -125,8 +123,7 @@ __global__ void __launch_bounds__(256) commit_overwrite_kernel(CacheView c, cons
 // One warp per (sequence, head, block): lanes 0-15 take rows 0-7, lanes 16-31
 // rows 8-15, each lane one 16-byte chunk (8 dims); halves combine by shuffle.
 __global__ void __launch_bounds__(256) update_summaries_kernel(CacheView c, int begin, int end) {
-  pdl_launch_dependents();
-  pdl_wait();
+  pdl_wait();  // no early launch of dependents: they may read the summaries and lengths written here
   const int b = blockIdx.z, h = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int blk = begin + blockIdx.x * 8 + warp;

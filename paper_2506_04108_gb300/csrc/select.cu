@@ -104,7 +104,7 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c,
   // over sequences (lengths out of range count as empty: top-n reports them)
   auto build_tables = [&]() {
     for (int b = tid; b < c.B; b += blockDim.x) {
-      const int T = c.seq_lens[b] + c.pending;
+      const int T = __ldcg(c.seq_lens + b) + c.pending;
       const bool bad = T < 0 || T > c.max_blocks * kBlock;
       sh_M[b] = bad ? 0 : (T + kBlock - 1) / kBlock;
       sh_T[b] = bad ? 0 : T;
@@ -144,49 +144,61 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c,
     blk0 = (r % per_head) * kPieceBlocks;
     nblk = min(kPieceBlocks, M - blk0);
   };
-  // Before the wait for the preceding kernel, prefetch this warp's pieces into
-  // L2 from the lengths as they are now (the append commit that may still be
-  // running changes at most the last block of a sequence; a stale length only
-  // misses or adds a prefetch, and addresses stay inside the summaries).
+  // The first pieces are fetched before the wait for the preceding kernel:
+  // every earlier writer of the summaries has completed by the time this
+  // kernel starts. The commits and the bulk summary build let their dependents
+  // launch only at exit, and this kernel (whose append writes them in a fused
+  // step) is always followed by a top-n kernel that lets its own dependents
+  // launch only after its wait. The lengths may still change under this
+  // prologue (the merge of a fused decode step advances them after letting
+  // its dependents launch), so they are read again after the wait, and if a
+  // block count differs the warps drain their copies and start over.
   build_tables();
-  {
-    const int total = sh_pref[c.B];
-    const int per = (total + gridDim.x - 1) / gridDim.x;
-    const int c0 = blockIdx.x * per, c1 = min(total, c0 + per);
-    const int ncta = max(0, c1 - c0);
-    const int nmine = ncta > warp ? (ncta - warp + kScoreWarps - 1) / kScoreWarps : 0;
-    if (lane == 0)
-      for (int k = 0; k < nmine; ++k) {
-        int b, h, blk0, nblk;
-        locate(c0 + warp + k * kScoreWarps, b, h, blk0, nblk);
-        bulk_prefetch_l2(c.summ + ((static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks + blk0) * 2 * kHeadDim,
-                         static_cast<uint32_t>(nblk) * 2 * kHeadDim * 2);
-      }
-  }
-  __syncthreads();  // the tables are rebuilt below
-  pdl_wait();
-  // The top-n kernel reads the lengths before its own wait: let it launch
-  // only now that the append commit (which advances them) has completed.
-  pdl_launch_dependents();
-  build_tables();
-  const int total = sh_pref[c.B];
-  const int per = (total + gridDim.x - 1) / gridDim.x;
-  const int c0 = blockIdx.x * per, c1 = min(total, c0 + per);
-  const int ncta = max(0, c1 - c0);
-  const int nmine = ncta > warp ? (ncta - warp + kScoreWarps - 1) / kScoreWarps : 0;
-
-  auto issue = [&](int k) {  // lane 0: this warp's k-th piece into stage k % kScoreStages
+  int total, per, c0, ncta, nmine, kbase = 0;  // kbase: copies issued before the current piece list
+  auto my_range = [&]() {
+    total = sh_pref[c.B];
+    per = (total + gridDim.x - 1) / gridDim.x;
+    c0 = blockIdx.x * per;
+    ncta = max(0, min(total, c0 + per) - c0);
+    nmine = ncta > warp ? (ncta - warp + kScoreWarps - 1) / kScoreWarps : 0;
+  };
+  my_range();
+  auto issue = [&](int k) {  // lane 0: this warp's k-th piece into stage (kbase + k) % kScoreStages
     int b, h, blk0, nblk;
     locate(c0 + warp + k * kScoreWarps, b, h, blk0, nblk);
-    const uint32_t bar = bar0 + 8 * (k % kScoreStages);
+    const uint32_t bar = bar0 + 8 * ((kbase + k) % kScoreStages);
     const uint32_t bytes = static_cast<uint32_t>(nblk) * 2 * kHeadDim * 2;
     mbar_arrive_expect_tx(bar, bytes);
-    bulk_load(ring_s + (k % kScoreStages) * kPieceBytes,
+    bulk_load(ring_s + ((kbase + k) % kScoreStages) * kPieceBytes,
               c.summ + ((static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks + blk0) * 2 * kHeadDim, bytes, bar);
   };
   __syncwarp();  // lane 0's barrier initialisation precedes every lane's use
   if (lane == 0)
     for (int k = 0; k < min(kScoreStages, nmine); ++k) issue(k);
+  const int issued_early = min(kScoreStages, nmine);
+  pdl_wait();
+  pdl_launch_dependents();  // the top-n kernel reads the lengths before its own wait
+  bool changed = false;
+  for (int b = tid; b < c.B; b += blockDim.x) {
+    const int T = __ldcg(c.seq_lens + b) + c.pending;
+    const bool bad = T < 0 || T > c.max_blocks * kBlock;
+    if ((bad ? 0 : (T + kBlock - 1) / kBlock) != sh_M[b]) changed = true;
+    sh_T[b] = bad ? 0 : T;
+  }
+  if (__syncthreads_or(changed)) {
+    bool drained = true;
+    if (lane == 0)
+      for (int k = 0; k < issued_early; ++k) drained = mbar_wait_bounded(bar0 + 8 * k, 0) && drained;
+    if (!__syncthreads_and(drained)) {
+      if (tid == 0) record_error(c.status, RESA_DEV_WAIT_TIMEOUT, -1);
+      return;
+    }
+    build_tables();
+    my_range();
+    kbase = issued_early;
+    if (lane == 0)
+      for (int k = 0; k < min(kScoreStages, nmine); ++k) issue(k);
+  }
 
   const int ch = lane & 15, half = lane >> 4;
   int cur_unit = -1, k_fail = -1;
@@ -194,7 +206,7 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c,
   uint32_t sg[4];
   uint4 ka = make_uint4(0, 0, 0, 0), va = ka;  // the appended token's key / value, this lane's 8 dims
   for (int k = 0; k < nmine; ++k) {
-    const int st = k % kScoreStages;
+    const int st = (kbase + k) % kScoreStages, par = ((kbase + k) / kScoreStages) & 1;
     int b, h, blk0, nblk;
     locate(c0 + warp + k * kScoreWarps, b, h, blk0, nblk);
     const int unit = b * c.Hkv + h;
@@ -232,14 +244,14 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c,
       }
     }
     int ok = 1;
-    if (lane == 0) ok = mbar_wait_bounded(bar0 + 8 * st, (k / kScoreStages) & 1) ? 1 : 0;
+    if (lane == 0) ok = mbar_wait_bounded(bar0 + 8 * st, par) ? 1 : 0;
     ok = __shfl_sync(0xffffffffu, ok, 0);
     if (!ok) {
       if (lane == 0) record_error(c.status, RESA_DEV_WAIT_TIMEOUT, unit);
       k_fail = k;
       break;
     }
-    mbar_try_wait(bar0 + 8 * st, (k / kScoreStages) & 1);
+    mbar_try_wait(bar0 + 8 * st, par);
     uint8_t* piece = ring + st * kPieceBytes;
     if (c.pending) {
       // Fused decode step: the appended token lands in block (T - 1) / 16.
@@ -305,7 +317,7 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c,
   // A warp that gave up may have copies in flight (pieces k_fail .. k_fail + 2):
   // wait for them (bounded) before the CTA exits.
   if (k_fail >= 0 && lane == 0) {
-    for (int k2 = k_fail; k2 < min(k_fail + kScoreStages, nmine); ++k2)
+    for (int k2 = kbase + k_fail; k2 < kbase + min(k_fail + kScoreStages, nmine); ++k2)
       (void)mbar_wait_bounded(bar0 + 8 * (k2 % kScoreStages), (k2 / kScoreStages) & 1);
   }
 }
@@ -380,13 +392,13 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
   __shared__ uint32_t cta_mm[2];  // this CTA's smallest and largest unforced key, read by peers
   namespace cg = cooperative_groups;
   cg::cluster_group cluster = cg::this_cluster();
-  pdl_launch_dependents();
   const int rank = static_cast<int>(cluster.block_rank());
   const int b = blockIdx.z, h = blockIdx.y;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   int32_t* out = indices + (static_cast<size_t>(b) * c.Hkv + h) * n_cap;
   const int T = __ldcg(c.seq_lens + b) + c.pending;  // final before the score kernel let this one launch
   pdl_wait();                            // the scores
+  pdl_launch_dependents();  // after the wait: see the score kernel
   if (T < 0 || T > c.max_blocks * kBlock) {  // the whole cluster takes this branch
     if (rank == 0 && tid == 0) {
       record_error(c.status, RESA_DEV_SEQ_LEN_RANGE, b);
@@ -626,12 +638,12 @@ __global__ void __launch_bounds__(kTopnCtaThreads, 1) topn_cta_kernel(CacheView 
   __shared__ int sh_pick[3];  // digit, rank left, whole bucket taken
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   for (int i = tid; i < 2 * 256; i += kTopnCtaThreads) (&hist[0][0])[i] = 0;
-  pdl_launch_dependents();
   const int h = blockIdx.x, b = blockIdx.y;
   int32_t* out = indices + (static_cast<size_t>(b) * c.Hkv + h) * n_cap;
   const int T = __ldcg(c.seq_lens + b) + c.pending;  // final before the score kernel let this one launch
   if (T < 0 || T > c.max_blocks * kBlock) {
     pdl_wait();
+    pdl_launch_dependents();
     if (tid == 0) {
       record_error(c.status, RESA_DEV_SEQ_LEN_RANGE, b);
       counts[b * c.Hkv + h] = 0;
@@ -643,6 +655,7 @@ __global__ void __launch_bounds__(kTopnCtaThreads, 1) topn_cta_kernel(CacheView 
   const int M = u.M, n = u.n, F = u.F, nf = u.nf, r = u.r;
   const float* sc = scores + (static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks;
   pdl_wait();  // the scores
+  pdl_launch_dependents();  // after the wait: see the score kernel
   uint32_t kmin = 0xFFFFFFFFu, kmax = 0u;
   for (int i0 = 0; i0 < M; i0 += 4 * kTopnCtaThreads) {  // four loads in flight per thread
     float v[4];
