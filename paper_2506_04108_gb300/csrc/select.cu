@@ -35,7 +35,7 @@ namespace resa {
 namespace {
 
 constexpr int kTopnCluster = 8;                                   // CTAs per (sequence, KV head)
-constexpr int kTopnThreads = 256;
+constexpr int kTopnThreads = 512;
 constexpr int kTopnWarps = kTopnThreads / 32;
 constexpr int kTopnSmemMax = 200 * 1024;                           // staged keys per CTA, bytes
 constexpr int kTopnCtaThreads = 512;                                // one-CTA form
@@ -354,51 +354,92 @@ __device__ __forceinline__ UnitBudget unit_budget(int T, double keep, int n_min,
   return u;
 }
 
-// Exclusive scan of one int per warp (kTopnWarps values, in place) by warp 0.
-__device__ __forceinline__ void scan_warp_totals(int* vals) {
+// Warp-wide inclusive scan of one int per lane.
+__device__ __forceinline__ int warp_incl_scan(int x) {
   const int lane = threadIdx.x & 31;
-  if (threadIdx.x < 32) {
-    const int v = lane < kTopnWarps ? vals[lane] : 0;
-    int x = v;
 #pragma unroll
-    for (int o = 1; o < kTopnWarps; o <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, x, o);
-      if (lane >= o) x += y;
-    }
-    if (lane < kTopnWarps) vals[lane] = x - v;
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
   }
+  return x;
 }
+
+// The radix digit holding the rem-th largest key, from a 256-bin histogram in
+// shared memory (every lane of the calling warp gets the answer): lane l owns
+// digits 255-8l ... 248-8l, read as two 16-byte loads.
+struct DigitPick {
+  int digit, rem, whole;  // digit, rank left within it, the whole bucket is taken
+};
+__device__ __forceinline__ DigitPick pick_digit(const int* hist, int rem) {
+  const int lane = threadIdx.x & 31;
+  const int4 a0 = reinterpret_cast<const int4*>(hist)[2 * (31 - lane)];
+  const int4 a1 = reinterpret_cast<const int4*>(hist)[2 * (31 - lane) + 1];
+  const int cn[8] = {a1.w, a1.z, a1.y, a1.x, a0.w, a0.z, a0.y, a0.x};
+  int sum = 0;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) sum += cn[j];
+  const int incl = warp_incl_scan(sum), excl = incl - sum;
+  const unsigned hit = __ballot_sync(0xffffffffu, excl < rem && rem <= incl);
+  const int src = hit ? __ffs(hit) - 1 : 0;  // 1 <= rem <= the histogram's total, so a lane holds it
+  DigitPick p{0, 0, 0};
+  if (lane == src) {
+    int cum = excl;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      if (cum + cn[j] >= rem) {
+        p.digit = 255 - 8 * lane - j;
+        p.rem = rem - cum;
+        p.whole = (rem - cum == cn[j]) ? 1 : 0;
+        break;
+      }
+      cum += cn[j];
+    }
+  }
+  p.digit = __shfl_sync(0xffffffffu, p.digit, src);
+  p.rem = __shfl_sync(0xffffffffu, p.rem, src);
+  p.whole = __shfl_sync(0xffffffffu, p.whole, src);
+  return p;
+}
+
+__device__ __forceinline__ void cluster_arrive() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
 
 // Cluster radix select, grid (kTopnCluster, KV head, sequence), one cluster
 // per (sequence, KV head). CTA r stages the order-preserving keys of blocks
 // [r * per, (r + 1) * per) in shared memory. Each 8-bit pass builds a local
 // histogram of the keys that still match the prefix; after one cluster
 // barrier every CTA sums the cluster's histograms through distributed shared
-// memory and finds the same digit (histograms are double-buffered by pass
-// parity, so one barrier per pass suffices). The select stops early when the
-// boundary bucket is taken whole. Then each CTA counts its keys above the
-// boundary and at it, reads the counts of the lower-ranked CTAs, and writes
-// its selected ids in ascending order (ties at the boundary to the lower id).
+// memory, and after one CTA barrier every warp finds the same digit
+// (histograms rotate through three buffers, each zeroed two passes after its
+// last remote read). The select stops early when the boundary bucket is taken
+// whole. Then each CTA counts its keys above the boundary and at it; every
+// warp reads the counts of the lower-ranked CTAs and of the lower warps and
+// writes its selected ids in ascending order (ties at the boundary to the
+// lower id). The closing cluster barrier is split: a CTA arrives after its
+// last remote read and waits only before it exits.
 __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const float* __restrict__ scores,
                                                             double keep, int n_min, int n_local,
                                                             int32_t* __restrict__ indices,
                                                             int32_t* __restrict__ counts, int n_cap) {
   extern __shared__ uint32_t keys[];
-  __shared__ int hist[2][256];
-  __shared__ int tot[256];
-  __shared__ int warp_a[kTopnWarps], warp_b[kTopnWarps];
-  __shared__ int sh_digit, sh_rem, sh_done, sh_eq_before, sh_sel_before;
-  __shared__ int cta_counts[2];  // keys above / at the boundary in this CTA, read by peers
-  __shared__ uint32_t cta_mm[2];  // this CTA's smallest and largest unforced key, read by peers
+  __shared__ __align__(16) int hist[3][256];
+  __shared__ __align__(16) int tot[256];
+  __shared__ int w_gt[kTopnWarps], w_eq[kTopnWarps];
+  __shared__ uint32_t w_mm[kTopnWarps][2];  // each warp's smallest and largest unforced key, read by peers
+  __shared__ int cta_counts[2];             // keys above / at the boundary in this CTA, read by peers
   namespace cg = cooperative_groups;
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = static_cast<int>(cluster.block_rank());
   const int b = blockIdx.z, h = blockIdx.y;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (int i = tid; i < 2 * 256; i += kTopnThreads) (&hist[0][0])[i] = 0;
   int32_t* out = indices + (static_cast<size_t>(b) * c.Hkv + h) * n_cap;
   const int T = __ldcg(c.seq_lens + b) + c.pending;  // final before the score kernel let this one launch
-  pdl_wait();                            // the scores
-  pdl_launch_dependents();  // after the wait: see the score kernel
+  pdl_wait();                                        // the scores
+  pdl_launch_dependents();                           // after the wait: see the score kernel
   if (T < 0 || T > c.max_blocks * kBlock) {  // the whole cluster takes this branch
     if (rank == 0 && tid == 0) {
       record_error(c.status, RESA_DEV_SEQ_LEN_RANGE, b);
@@ -414,53 +455,48 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
   const float* sc = scores + (static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks + lo;
   const int f_loc = F - lo;  // this CTA's ids >= f_loc are forced
   uint32_t kmin = 0xFFFFFFFFu, kmax = 0u;
-  for (int i0 = 0; i0 < cnt; i0 += 4 * kTopnThreads) {  // four loads in flight per thread
-    float v[4];
+  constexpr int kLoads = 8;  // loads in flight per thread
+  for (int i0 = 0; i0 < cnt; i0 += kLoads * kTopnThreads) {
+    float v[kLoads];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int i = i0 + u * kTopnThreads + tid;
-      v[u] = i < cnt ? sc[i] : 0.f;
+    for (int k = 0; k < kLoads; ++k) {
+      const int i = i0 + k * kTopnThreads + tid;
+      v[k] = i < cnt ? sc[i] : 0.f;
     }
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int i = i0 + u * kTopnThreads + tid;
+    for (int k = 0; k < kLoads; ++k) {
+      const int i = i0 + k * kTopnThreads + tid;
       if (i < cnt) {
-        const uint32_t k = score_key(v[u]);
-        keys[i] = k;
+        const uint32_t key = score_key(v[k]);
+        keys[i] = key;
         if (i < f_loc) {
-          kmin = min(kmin, k);
-          kmax = max(kmax, k);
+          kmin = min(kmin, key);
+          kmax = max(kmax, key);
         }
       }
     }
   }
-  const int cnt_round = (cnt + 31) / 32 * 32;
-  // extreme unforced keys of the unit: CTA reduction, then across the cluster
+  // extreme unforced keys of the unit: per warp, then every warp reduces the
+  // cluster's kTopnCluster x kTopnWarps partials
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     kmin = min(kmin, __shfl_xor_sync(0xffffffffu, kmin, o));
     kmax = max(kmax, __shfl_xor_sync(0xffffffffu, kmax, o));
   }
   if (lane == 0) {
-    warp_a[warp] = static_cast<int>(kmin);
-    warp_b[warp] = static_cast<int>(kmax);
+    w_mm[warp][0] = kmin;
+    w_mm[warp][1] = kmax;
   }
-  __syncthreads();
-  if (tid == 0) {
-    uint32_t a = 0xFFFFFFFFu, z = 0u;
-    for (int w = 0; w < kTopnWarps; ++w) {
-      a = min(a, static_cast<uint32_t>(warp_a[w]));
-      z = max(z, static_cast<uint32_t>(warp_b[w]));
-    }
-    cta_mm[0] = a;
-    cta_mm[1] = z;
-  }
-  cluster.sync();  // every CTA's extremes are visible
-#pragma unroll
-  for (int q = 0; q < kTopnCluster; ++q) {
-    const uint32_t* pm = cluster.map_shared_rank(cta_mm, q);
+  cluster.sync();  // every warp's extremes and every CTA's keys are visible
+  for (int e = lane; e < kTopnCluster * kTopnWarps; e += 32) {
+    const uint32_t* pm = cluster.map_shared_rank(&w_mm[0][0], e / kTopnWarps) + 2 * (e % kTopnWarps);
     kmin = min(kmin, pm[0]);
     kmax = max(kmax, pm[1]);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    kmin = min(kmin, __shfl_xor_sync(0xffffffffu, kmin, o));
+    kmax = max(kmax, __shfl_xor_sync(0xffffffffu, kmax, o));
   }
 
   // ---- radix select of the r-th largest v = key - kmin among blocks [0, F) ----
@@ -474,58 +510,26 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
     int shift = max(bits - 8, 0), width = bits - shift;
     for (int pass = 0;; ++pass) {
       const uint32_t dmask = (1u << width) - 1u;
-      int* hb = hist[pass & 1];
-      hb[tid] = 0;
-      __syncthreads();
-      for (int i = tid; i < cnt_round; i += kTopnThreads) {
-        uint32_t d = 0x100u;  // sentinel: not counted
-        if (i < cnt && i < f_loc) {
-          const uint32_t v = keys[i] - kmin;
-          if ((v & pmask) == prefix) d = (v >> shift) & dmask;
-        }
-        const unsigned peers = __match_any_sync(0xffffffffu, d);
-        if (d != 0x100u && lane == __ffs(peers) - 1) atomicAdd(&hb[d], __popc(peers));
+      int* hb = hist[pass % 3];
+      // the buffer of the next pass: its last remote reads were two passes ago
+      for (int i = tid; i < 256; i += kTopnThreads) hist[(pass + 1) % 3][i] = 0;
+      for (int i = tid; i < min(cnt, f_loc); i += kTopnThreads) {
+        const uint32_t v = keys[i] - kmin;
+        if ((v & pmask) == prefix) atomicAdd(&hb[(v >> shift) & dmask], 1);
       }
       cluster.sync();  // every CTA's histogram of this pass is complete and visible
-      int t = 0;
+      for (int bin = tid; bin < 256; bin += kTopnThreads) {
+        int t = 0;
 #pragma unroll
-      for (int r = 0; r < kTopnCluster; ++r) t += cluster.map_shared_rank(hb, r)[tid];
-      tot[tid] = t;
-      __syncthreads();
-      if (warp == 0) {
-        // lane l owns digits 255-8l ... 248-8l (descending)
-        int cn[8], sum = 0;
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          cn[j] = tot[255 - 8 * lane - j];
-          sum += cn[j];
-        }
-        int incl = sum;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const int y = __shfl_up_sync(0xffffffffu, incl, o);
-          if (lane >= o) incl += y;
-        }
-        const int excl = incl - sum;
-        if (excl < rem && rem <= incl) {
-          int cum = excl;
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            if (cum + cn[j] >= rem) {
-              sh_digit = 255 - 8 * lane - j;
-              sh_rem = rem - cum;
-              sh_done = (rem - cum == cn[j]) ? 1 : 0;  // the whole bucket is taken
-              break;
-            }
-            cum += cn[j];
-          }
-        }
+        for (int q = 0; q < kTopnCluster; ++q) t += cluster.map_shared_rank(hb, q)[bin];
+        tot[bin] = t;
       }
       __syncthreads();
-      prefix |= static_cast<uint32_t>(sh_digit) << shift;
+      const DigitPick pk = pick_digit(tot, rem);  // the same in every warp and every CTA
+      prefix |= static_cast<uint32_t>(pk.digit) << shift;
       pmask |= dmask << shift;
-      rem = sh_rem;
-      if (sh_done || shift == 0) break;  // identical decision in every CTA of the cluster
+      rem = pk.rem;
+      if (pk.whole || shift == 0) break;
       width = min(8, shift);
       shift -= width;
     }
@@ -549,75 +553,67 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
   };
 
   // ---- ordered compaction: warps own contiguous id ranges of the CTA ----
-  const int per_warp = (cnt_round / 32 + kTopnWarps - 1) / kTopnWarps * 32;
+  const int per_warp = ((cnt + 31) / 32 + kTopnWarps - 1) / kTopnWarps * 32;
   const int w0 = warp * per_warp, w1 = min(cnt, w0 + per_warp);
   int gt = 0, eq = 0;
-  if (n > 0) {
-    for (int i0 = w0; i0 < w0 + per_warp; i0 += 32) {
-      const int i = i0 + lane;
-      bool is_gt, is_eq;
-      classify(i, i < w1, is_gt, is_eq);
-      gt += __popc(__ballot_sync(0xffffffffu, is_gt));
-      eq += __popc(__ballot_sync(0xffffffffu, is_eq));
-    }
+  for (int i0 = w0; i0 < w1; i0 += 32) {
+    bool is_gt, is_eq;
+    classify(i0 + lane, i0 + lane < w1, is_gt, is_eq);
+    gt += __popc(__ballot_sync(0xffffffffu, is_gt));
+    eq += __popc(__ballot_sync(0xffffffffu, is_eq));
   }
   if (lane == 0) {
-    warp_a[warp] = eq;
-    warp_b[warp] = gt;
+    w_gt[warp] = gt;
+    w_eq[warp] = eq;
   }
   __syncthreads();
-  if (tid == 0) {
-    int g2 = 0, e2 = 0;
-    for (int w = 0; w < kTopnWarps; ++w) {
-      g2 += warp_b[w];
-      e2 += warp_a[w];
+  // this CTA's totals (every warp computes them; warp 0 publishes them)
+  const int g_l = lane < kTopnWarps ? w_gt[lane] : 0, e_l = lane < kTopnWarps ? w_eq[lane] : 0;
+  const int g_in = warp_incl_scan(g_l), e_in = warp_incl_scan(e_l);
+  if (warp == 0) {
+    const int gt_cta = __shfl_sync(0xffffffffu, g_in, 31), eq_cta = __shfl_sync(0xffffffffu, e_in, 31);
+    if (lane == 0) {
+      cta_counts[0] = gt_cta;
+      cta_counts[1] = eq_cta;
     }
-    cta_counts[0] = g2;
-    cta_counts[1] = e2;
   }
   cluster.sync();  // every CTA's counts are visible
-  if (tid == 0) {
-    int eq_before = 0, sel_before = 0;
-    for (int r = 0; r < rank; ++r) {
-      const int* pc = cluster.map_shared_rank(cta_counts, r);
-      const int g2 = pc[0], e2 = pc[1];
-      sel_before += g2 + max(0, min(e2, take_eq - eq_before));
-      eq_before += e2;
-    }
-    sh_eq_before = eq_before;
-    sh_sel_before = sel_before;
+  // lower-ranked CTAs: lane q < rank reads CTA q's counts
+  int gq = 0, eqq = 0;
+  if (lane < rank) {
+    const int* pc = cluster.map_shared_rank(cta_counts, lane);
+    gq = pc[0];
+    eqq = pc[1];
   }
-  __syncthreads();
-  scan_warp_totals(warp_a);  // exclusive prefix of equal keys per warp
-  __syncthreads();
-  if (lane == 0) {
-    const int eq_b = sh_eq_before + warp_a[warp];
-    warp_b[warp] = gt + max(0, min(eq, take_eq - eq_b));
-  }
-  __syncthreads();
-  scan_warp_totals(warp_b);  // exclusive prefix of selected ids per warp
-  __syncthreads();
-  if (n > 0) {
-    int eq_seen = sh_eq_before + warp_a[warp];
-    int pos = sh_sel_before + warp_b[warp];
-    for (int i0 = w0; i0 < w0 + per_warp; i0 += 32) {
-      const int i = i0 + lane;
-      bool is_gt, is_eq;
-      classify(i, i < w1, is_gt, is_eq);
-      const unsigned eqm = __ballot_sync(0xffffffffu, is_eq);
-      const int my_eq_rank = eq_seen + __popc(eqm & ((1u << lane) - 1u));
-      const bool sel = is_gt || (is_eq && my_eq_rank < take_eq);
-      const unsigned selm = __ballot_sync(0xffffffffu, sel);
-      if (sel) out[pos + __popc(selm & ((1u << lane) - 1u))] = lo + i;
-      eq_seen += __popc(eqm);
-      pos += __popc(selm);
-    }
+  cluster_arrive();  // no remote reads after this point
+  const int eq_incl = warp_incl_scan(eqq);
+  const int sel_q = gq + max(0, min(eqq, take_eq - (eq_incl - eqq)));
+  int sel_before = sel_q;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) sel_before += __shfl_xor_sync(0xffffffffu, sel_before, o);
+  const int eq_before = __shfl_sync(0xffffffffu, eq_incl, 31);
+  // lower warps of this CTA
+  const int e_ex = e_in - e_l;
+  const int s_l = g_l + max(0, min(e_l, take_eq - (eq_before + e_ex)));
+  const int s_in = warp_incl_scan(s_l);
+  int eq_seen = eq_before + __shfl_sync(0xffffffffu, e_ex, warp);
+  int pos = sel_before + __shfl_sync(0xffffffffu, s_in - s_l, warp);
+  for (int i0 = w0; i0 < w1; i0 += 32) {
+    const int i = i0 + lane;
+    bool is_gt, is_eq;
+    classify(i, i < w1, is_gt, is_eq);
+    const unsigned eqm = __ballot_sync(0xffffffffu, is_eq);
+    const int my_eq_rank = eq_seen + __popc(eqm & ((1u << lane) - 1u));
+    const bool sel = is_gt || (is_eq && my_eq_rank < take_eq);
+    const unsigned selm = __ballot_sync(0xffffffffu, sel);
+    if (sel) out[pos + __popc(selm & ((1u << lane) - 1u))] = lo + i;
+    eq_seen += __popc(eqm);
+    pos += __popc(selm);
   }
   for (int i = n + rank * kTopnThreads + tid; i < n_cap; i += kTopnCluster * kTopnThreads) out[i] = -1;
   if (rank == 0 && tid == 0) counts[b * c.Hkv + h] = n;
-  cluster.sync();  // no CTA leaves while a peer may still read its counts
+  cluster_wait();  // no CTA leaves while a peer may still read its shared memory
 }
-
 
 // One-CTA radix select, grid (KV head, sequence), for caches of up to
 // kTopnCtaMaxBlocks blocks per sequence: the same selection as topn_kernel
@@ -711,32 +707,11 @@ __global__ void __launch_bounds__(kTopnCtaThreads, 1) topn_cta_kernel(CacheView 
       }
       __syncthreads();  // this pass's histogram is complete
       if (warp == 0) {
-        // lane l owns digits 255-8l ... 248-8l (descending): two 16-byte loads
-        const int4 a0 = reinterpret_cast<const int4*>(hb)[2 * (31 - lane)];
-        const int4 a1 = reinterpret_cast<const int4*>(hb)[2 * (31 - lane) + 1];
-        const int cn[8] = {a1.w, a1.z, a1.y, a1.x, a0.w, a0.z, a0.y, a0.x};
-        int sum = 0;
-#pragma unroll
-        for (int j = 0; j < 8; ++j) sum += cn[j];
-        int incl = sum;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const int y = __shfl_up_sync(0xffffffffu, incl, o);
-          if (lane >= o) incl += y;
-        }
-        const int excl = incl - sum;
-        if (excl < rem && rem <= incl) {
-          int cum = excl;
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            if (cum + cn[j] >= rem) {
-              sh_pick[0] = 255 - 8 * lane - j;
-              sh_pick[1] = rem - cum;
-              sh_pick[2] = (rem - cum == cn[j]) ? 1 : 0;  // the whole bucket is taken
-              break;
-            }
-            cum += cn[j];
-          }
+        const DigitPick pk = pick_digit(hb, rem);
+        if (lane == 0) {
+          sh_pick[0] = pk.digit;
+          sh_pick[1] = pk.rem;
+          sh_pick[2] = pk.whole;
         }
       }
       __syncthreads();  // the digit is visible
