@@ -653,15 +653,17 @@ __global__ void __launch_bounds__(kTopnCtaThreads, 1) topn_cta_kernel(CacheView 
   pdl_wait();  // the scores
   pdl_launch_dependents();  // after the wait: see the score kernel
   uint32_t kmin = 0xFFFFFFFFu, kmax = 0u;
-  for (int i0 = 0; i0 < M; i0 += 4 * kTopnCtaThreads) {  // four loads in flight per thread
-    float v[4];
+  // one round of loads for up to 4096 blocks (a unit of 32K tokens holds 2049)
+  constexpr int kLoads = 8;
+  for (int i0 = 0; i0 < M; i0 += kLoads * kTopnCtaThreads) {
+    float v[kLoads];
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
+    for (int k = 0; k < kLoads; ++k) {
       const int i = i0 + k * kTopnCtaThreads + tid;
       v[k] = i < M ? sc[i] : 0.f;
     }
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
+    for (int k = 0; k < kLoads; ++k) {
       const int i = i0 + k * kTopnCtaThreads + tid;
       if (i < M) {
         const uint32_t key = score_key(v[k]);

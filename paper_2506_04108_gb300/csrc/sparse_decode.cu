@@ -272,13 +272,15 @@ __global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid
     red[(warp * 8 + hB) * kHeadDim + dB] = acc[mt][3] * fB;
   }
   __syncthreads();
-  const int t = threadIdx.x;  // one output dim per thread
+  const int t = threadIdx.x;
   for (int hh = 0; hh < c.g; ++hh) {
-    float v = 0.f;
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w) v += red[(w * 8 + hh) * kHeadDim + t];
     const size_t row = static_cast<size_t>(b) * c.Hq + h * c.g + hh;
-    a.o_part[(row * a.splits + s) * kHeadDim + t] = v;
+    for (int dd = t; dd < kHeadDim; dd += kWarps * 32) {  // output dims of this thread
+      float v = 0.f;
+#pragma unroll
+      for (int w = 0; w < kWarps; ++w) v += red[(w * 8 + hh) * kHeadDim + dd];
+      a.o_part[(row * a.splits + s) * kHeadDim + dd] = v;
+    }
   }
   if (t < c.g) {
     float Mt = kNegInf;
