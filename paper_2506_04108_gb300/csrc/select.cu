@@ -1,6 +1,6 @@
 // Block selection (Section 2.1 "Block Selection"; Eq. 4 and Eq. 5).
 //
-// score_kernel  persistent, one CTA per SM: each of its 16 warps streams 4 KB
+// score_kernel  persistent, one CTA per SM: each of its 16 warps streams 6 KB
 //               pieces of the block summaries with its own bulk copies through
 //               its own shared-memory ring and scores them with the pooled
 //               query of the piece's GQA group (mean of the g heads, fp32); a
@@ -69,19 +69,20 @@ __device__ __forceinline__ float quest_term8(const float* qa, const uint32_t* sg
 }
 
 // Persistent score kernel: one CTA per SM. The (sequence, KV head) units'
-// summaries are cut into pieces of 8 blocks (4 KB, contiguous); CTA x owns
+// summaries are cut into pieces of 12 blocks (6 KB, contiguous); CTA x owns
 // the piece range [x * per, (x + 1) * per) of the flattened piece list and
 // its warp w takes every 16th piece of it (w, w + 16, ...). Each warp streams
 // its pieces with 1-D bulk copies issued by its own lane 0 through its own
-// 3-stage shared-memory ring: copies issued by one thread complete one after
-// another, so sixteen independent issuers keep enough bytes in flight per SM.
+// 2-stage shared-memory ring: copies issued by one thread complete one after
+// another, so sixteen independent issuers keep enough bytes in flight per SM
+// (measured: 6 KB pieces in 2 stages beat 4 KB in 3 and 8 KB with 12 warps).
 // A half-warp scores one block, a lane one 16-byte piece (8 dims) of k_min
 // and k_max, and the 128-dim sum ends in a fixed-order 16-lane butterfly.
 constexpr int kScoreWarps = 16;
-constexpr int kScoreStages = 3;                                    // pieces in flight per warp
+constexpr int kScoreStages = 2;                                    // pieces in flight per warp
 constexpr int kMaxBatch = 1024;  // sequences per call supported by the score kernel
-constexpr int kPieceBlocks = 8;
-constexpr int kPieceBytes = kPieceBlocks * 2 * kHeadDim * 2;       // 4 KB
+constexpr int kPieceBlocks = 12;
+constexpr int kPieceBytes = kPieceBlocks * 2 * kHeadDim * 2;       // 6 KB
 constexpr int kScoreRing = kScoreWarps * kScoreStages * kPieceBytes;  // 192 KB
 constexpr int kScoreSmem = kScoreRing + kScoreWarps * kScoreStages * 8;
 
@@ -314,7 +315,7 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c,
       issue(k + kScoreStages);
     }
   }
-  // A warp that gave up may have copies in flight (pieces k_fail .. k_fail + 2):
+  // A warp that gave up may have copies in flight (pieces k_fail .. k_fail + kScoreStages - 1):
   // wait for them (bounded) before the CTA exits.
   if (k_fail >= 0 && lane == 0) {
     for (int k2 = kbase + k_fail; k2 < kbase + min(k_fail + kScoreStages, nmine); ++k2)
