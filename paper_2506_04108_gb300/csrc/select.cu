@@ -84,15 +84,18 @@ constexpr int kMaxBatch = 1024;  // sequences per call supported by the score ke
 constexpr int kPieceBlocks = 12;
 constexpr int kPieceBytes = kPieceBlocks * 2 * kHeadDim * 2;       // 6 KB
 constexpr int kScoreRing = kScoreWarps * kScoreStages * kPieceBytes;  // 192 KB
-constexpr int kScoreSmem = kScoreRing + kScoreWarps * kScoreStages * 8;
+constexpr int kScoreSmem = kScoreRing + kScoreWarps * kScoreStages * 8;  // + score_table_bytes(B)
+constexpr int score_table_bytes(int B) { return (3 * B + 1) * static_cast<int>(sizeof(int)); }
 
 __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c, const uint16_t* __restrict__ q,
                                                                     float* __restrict__ scores) {
   extern __shared__ __align__(1024) uint8_t smem[];
-  // per-sequence block counts and the piece prefix over (sequence, head) units
-  __shared__ int sh_M[kMaxBatch];
-  __shared__ int sh_T[kMaxBatch];
-  __shared__ int sh_pref[kMaxBatch + 1];
+  // per-sequence block counts and the piece prefix over (sequence, head)
+  // units, after the rings and their barriers (sized by the batch, so that
+  // the top-n CTAs launched early fit beside this CTA)
+  int* sh_M = reinterpret_cast<int*>(smem + kScoreSmem);
+  int* sh_T = sh_M + c.B;
+  int* sh_pref = sh_T + c.B;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   uint8_t* ring = smem + warp * kScoreStages * kPieceBytes;
   const uint32_t ring_s = smem_u32(ring);
@@ -408,34 +411,76 @@ __device__ __forceinline__ void cluster_arrive() {
 }
 __device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
 
+// Distributed shared memory pushes: the shared::cluster address of `a` (an
+// address of this CTA's shared memory) in cluster CTA `rank`, and stores into
+// a peer's shared memory that complete on the peer's mbarrier (transaction
+// bytes), so the receiver needs no cluster-scope fence to read them.
+__device__ __forceinline__ uint32_t peer_addr(uint32_t a, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void push_v4(uint32_t dst, const int4& v, uint32_t bar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.s32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(dst),
+               "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w), "r"(bar)
+               : "memory");
+}
+__device__ __forceinline__ void push_v2(uint32_t dst, uint32_t x, uint32_t y, uint32_t bar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.b32 [%0], {%1, %2}, [%3];" ::"r"(dst),
+               "r"(x), "r"(y), "r"(bar)
+               : "memory");
+}
+
 // Cluster radix select, grid (kTopnCluster, KV head, sequence), one cluster
 // per (sequence, KV head). CTA r stages the order-preserving keys of blocks
-// [r * per, (r + 1) * per) in shared memory. Each 8-bit pass builds a local
-// histogram of the keys that still match the prefix; after one cluster
-// barrier every CTA sums the cluster's histograms through distributed shared
-// memory, and after one CTA barrier every warp finds the same digit
-// (histograms rotate through three buffers, each zeroed two passes after its
-// last remote read). The select stops early when the boundary bucket is taken
-// whole. Then each CTA counts its keys above the boundary and at it; every
-// warp reads the counts of the lower-ranked CTAs and of the lower warps and
-// writes its selected ids in ascending order (ties at the boundary to the
-// lower id). The closing cluster barrier is split: a CTA arrives after its
-// last remote read and waits only before it exits.
-__global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const float* __restrict__ scores,
+// [r * per, (r + 1) * per) in shared memory. Every exchange between the CTAs
+// is a push: a CTA stores its part (extremes, each pass's 256-bin histogram,
+// its selected counts) into every CTA's receive buffer with stores that
+// complete on the receiver's mbarrier, and each CTA waits on its own barrier
+// for all eight parts. Only the barriers' initialisation needs a cluster
+// barrier, whose arrive is issued at entry and whose wait comes before the
+// first push. Each 8-bit pass builds a local histogram of the keys that still
+// match the prefix; after the exchange every CTA sums the eight histograms
+// and after one CTA barrier every warp finds the same digit (receive buffers
+// alternate between passes: a CTA pushes pass p + 2 only after it received
+// every CTA's pass p + 1, which each sent after reading its pass p buffer).
+// The select stops early when the boundary bucket is taken whole. Then each
+// CTA counts its keys above the boundary and at it; every warp reads the
+// counts of the lower-ranked CTAs and of the lower warps and writes its
+// selected ids in ascending order (ties at the boundary to the lower id). A
+// CTA leaves once it holds all its parts: no peer writes to it afterwards.
+// A wait that runs out records RESA_DEV_WAIT_TIMEOUT; the thread then writes
+// no ids and waits at a cluster barrier (which completes once every other
+// thread has arrived or exited) before it leaves.
+// 40 registers (3 CTAs per SM): a CTA launched early then fits beside the
+// persistent score CTA (88 registers x 512 threads), so its prologue runs
+// before the scores are complete.
+__global__ void __launch_bounds__(kTopnThreads, 3) topn_kernel(CacheView c, const float* __restrict__ scores,
                                                             double keep, int n_min, int n_local,
                                                             int32_t* __restrict__ indices,
                                                             int32_t* __restrict__ counts, int n_cap) {
+  static_assert(kTopnThreads >= kTopnCluster * 32, "one 16-byte push per thread of the first 8 warps and pass");
+  static_assert(kTopnSmemMax / sizeof(uint32_t) <= 0xFFFF, "a CTA's bin count fits 16 bits");
   extern __shared__ uint32_t keys[];
-  __shared__ __align__(16) int hist[3][256];
+  __shared__ __align__(16) int hist[2][256];                     // local histogram of pass p in hist[p & 1]
+  __shared__ __align__(16) uint16_t recv[2][kTopnCluster][256];  // every CTA's histogram of pass p in recv[p & 1]
   __shared__ __align__(16) int tot[256];
+  __shared__ __align__(8) uint32_t recv_mm[kTopnCluster][2];  // every CTA's smallest and largest unforced key
+  __shared__ __align__(8) int recv_cnt[kTopnCluster][2];      // every CTA's keys above / at the boundary
+  __shared__ __align__(8) uint64_t bars[4];                   // passes (2, alternating), extremes, counts
   __shared__ int w_gt[kTopnWarps], w_eq[kTopnWarps];
-  __shared__ uint32_t w_mm[kTopnWarps][2];  // each warp's smallest and largest unforced key, read by peers
-  __shared__ int cta_counts[2];             // keys above / at the boundary in this CTA, read by peers
-  namespace cg = cooperative_groups;
-  cg::cluster_group cluster = cg::this_cluster();
-  const int rank = static_cast<int>(cluster.block_rank());
+  __shared__ uint32_t w_mm[kTopnWarps][2];
+  uint32_t rank;
+  asm("mov.u32 %0, %%cluster_ctarank;" : "=r"(rank));
   const int b = blockIdx.z, h = blockIdx.y;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const uint32_t bar0 = smem_u32(&bars[0]);
+  if (tid == 0) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) mbar_init(bar0 + 8 * i, 1);
+    fence_mbar_init();
+  }
+  cluster_arrive();  // the barriers are initialised (waited for before the first push)
   for (int i = tid; i < 2 * 256; i += kTopnThreads) (&hist[0][0])[i] = 0;
   int32_t* out = indices + (static_cast<size_t>(b) * c.Hkv + h) * n_cap;
   const int T = __ldcg(c.seq_lens + b) + c.pending;  // final before the score kernel let this one launch
@@ -446,13 +491,14 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
       record_error(c.status, RESA_DEV_SEQ_LEN_RANGE, b);
       counts[b * c.Hkv + h] = 0;
     }
-    for (int i = rank * kTopnThreads + tid; i < n_cap; i += kTopnCluster * kTopnThreads) out[i] = -1;
+    for (int i = static_cast<int>(rank) * kTopnThreads + tid; i < n_cap; i += kTopnCluster * kTopnThreads) out[i] = -1;
+    cluster_wait();
     return;
   }
   const UnitBudget u = unit_budget(T, keep, n_min, n_local, n_cap, c.status, b * c.Hkv + h, rank == 0 && tid == 0);
   const int M = u.M, n = u.n, F = u.F, nf = u.nf, r = u.r;
   const int per = (M + kTopnCluster - 1) / kTopnCluster;
-  const int lo = rank * per, cnt = max(0, min(M, lo + per) - lo);
+  const int lo = static_cast<int>(rank) * per, cnt = max(0, min(M, lo + per) - lo);
   const float* sc = scores + (static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks + lo;
   const int f_loc = F - lo;  // this CTA's ids >= f_loc are forced
   uint32_t kmin = 0xFFFFFFFFu, kmax = 0u;
@@ -477,8 +523,7 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
       }
     }
   }
-  // extreme unforced keys of the unit: per warp, then every warp reduces the
-  // cluster's kTopnCluster x kTopnWarps partials
+  // extreme unforced keys: per warp, per CTA (warp 0), then pushed to every CTA
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     kmin = min(kmin, __shfl_xor_sync(0xffffffffu, kmin, o));
@@ -488,12 +533,26 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
     w_mm[warp][0] = kmin;
     w_mm[warp][1] = kmax;
   }
-  cluster.sync();  // every warp's extremes and every CTA's keys are visible
-  for (int e = lane; e < kTopnCluster * kTopnWarps; e += 32) {
-    const uint32_t* pm = cluster.map_shared_rank(&w_mm[0][0], e / kTopnWarps) + 2 * (e % kTopnWarps);
-    kmin = min(kmin, pm[0]);
-    kmax = max(kmax, pm[1]);
+  __syncthreads();  // the keys and every warp's extremes are visible
+  cluster_wait();   // every CTA's barriers are initialised
+  // `failed` (a wait ran out) is made uniform over the CTA at its barriers;
+  // a CTA that failed pushes nothing more and skips its remaining waits.
+  bool failed = false;
+  if (warp == 0) {
+    kmin = lane < kTopnWarps ? w_mm[lane][0] : 0xFFFFFFFFu;
+    kmax = lane < kTopnWarps ? w_mm[lane][1] : 0u;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      kmin = min(kmin, __shfl_xor_sync(0xffffffffu, kmin, o));
+      kmax = max(kmax, __shfl_xor_sync(0xffffffffu, kmax, o));
+    }
+    if (lane < kTopnCluster)
+      push_v2(peer_addr(smem_u32(&recv_mm[rank][0]), lane), kmin, kmax, peer_addr(bar0 + 16, lane));
+    if (lane == 0) mbar_arrive_expect_tx(bar0 + 16, kTopnCluster * 8);
   }
+  failed |= !mbar_wait_bounded(bar0 + 16, 0);
+  kmin = lane < kTopnCluster ? recv_mm[lane][0] : 0xFFFFFFFFu;
+  kmax = lane < kTopnCluster ? recv_mm[lane][1] : 0u;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     kmin = min(kmin, __shfl_xor_sync(0xffffffffu, kmin, o));
@@ -509,23 +568,33 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
   if (r > 0 && r < F) {
     const int bits = 32 - __clz(static_cast<int>(kmax - kmin));  // significant bits of v
     int shift = max(bits - 8, 0), width = bits - shift;
+    const int dst = tid >> 5, part = tid & 31;  // threads < 256: bins [8 part, 8 part + 8) to CTA dst
     for (int pass = 0;; ++pass) {
       const uint32_t dmask = (1u << width) - 1u;
-      int* hb = hist[pass % 3];
-      // the buffer of the next pass: its last remote reads were two passes ago
-      for (int i = tid; i < 256; i += kTopnThreads) hist[(pass + 1) % 3][i] = 0;
+      int* hb = hist[pass & 1];
       for (int i = tid; i < min(cnt, f_loc); i += kTopnThreads) {
         const uint32_t v = keys[i] - kmin;
         if ((v & pmask) == prefix) atomicAdd(&hb[(v >> shift) & dmask], 1);
       }
-      cluster.sync();  // every CTA's histogram of this pass is complete and visible
-      for (int bin = tid; bin < 256; bin += kTopnThreads) {
+      failed = __syncthreads_or(failed);  // this CTA's histogram of the pass is complete
+      if (!failed) {
+        const uint32_t bar = bar0 + 8 * (pass & 1);
+        if (tid < kTopnCluster * 32) {
+          const int4 a = reinterpret_cast<const int4*>(hb)[2 * part], e = reinterpret_cast<const int4*>(hb)[2 * part + 1];
+          const int4 v = make_int4(a.x | (a.y << 16), a.z | (a.w << 16), e.x | (e.y << 16), e.z | (e.w << 16));
+          push_v4(peer_addr(smem_u32(&recv[pass & 1][rank][8 * part]), dst), v, peer_addr(bar, dst));
+        }
+        if (tid == 0) mbar_arrive_expect_tx(bar, kTopnCluster * 256 * sizeof(uint16_t));
+        failed = !mbar_wait_bounded(bar, (pass >> 1) & 1);
+      }
+      if (tid < 256) {
         int t = 0;
 #pragma unroll
-        for (int q = 0; q < kTopnCluster; ++q) t += cluster.map_shared_rank(hb, q)[bin];
-        tot[bin] = t;
+        for (int q = 0; q < kTopnCluster; ++q) t += recv[pass & 1][q][tid];
+        tot[tid] = t;
       }
-      __syncthreads();
+      failed = __syncthreads_or(failed);  // the cluster's histogram is visible; every thread has pushed this pass
+      for (int i = tid; i < 256; i += kTopnThreads) hb[i] = 0;  // for pass + 2 (the next barrier orders it)
       const DigitPick pk = pick_digit(tot, rem);  // the same in every warp and every CTA
       prefix |= static_cast<uint32_t>(pk.digit) << shift;
       pmask |= dmask << shift;
@@ -567,26 +636,26 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
     w_gt[warp] = gt;
     w_eq[warp] = eq;
   }
-  __syncthreads();
-  // this CTA's totals (every warp computes them; warp 0 publishes them)
+  failed = __syncthreads_or(failed);
+  // this CTA's totals (every warp computes them; warp 0 pushes them to every CTA)
   const int g_l = lane < kTopnWarps ? w_gt[lane] : 0, e_l = lane < kTopnWarps ? w_eq[lane] : 0;
   const int g_in = warp_incl_scan(g_l), e_in = warp_incl_scan(e_l);
-  if (warp == 0) {
-    const int gt_cta = __shfl_sync(0xffffffffu, g_in, 31), eq_cta = __shfl_sync(0xffffffffu, e_in, 31);
-    if (lane == 0) {
-      cta_counts[0] = gt_cta;
-      cta_counts[1] = eq_cta;
+  if (!failed) {
+    if (warp == 0) {
+      const int gt_cta = __shfl_sync(0xffffffffu, g_in, 31), eq_cta = __shfl_sync(0xffffffffu, e_in, 31);
+      if (lane < kTopnCluster)
+        push_v2(peer_addr(smem_u32(&recv_cnt[rank][0]), lane), static_cast<uint32_t>(gt_cta),
+                static_cast<uint32_t>(eq_cta), peer_addr(bar0 + 24, lane));
+      if (lane == 0) mbar_arrive_expect_tx(bar0 + 24, kTopnCluster * 8);
     }
+    failed = __any_sync(0xffffffffu, !mbar_wait_bounded(bar0 + 24, 0));
   }
-  cluster.sync();  // every CTA's counts are visible
   // lower-ranked CTAs: lane q < rank reads CTA q's counts
   int gq = 0, eqq = 0;
-  if (lane < rank) {
-    const int* pc = cluster.map_shared_rank(cta_counts, lane);
-    gq = pc[0];
-    eqq = pc[1];
+  if (lane < static_cast<int>(rank)) {
+    gq = recv_cnt[lane][0];
+    eqq = recv_cnt[lane][1];
   }
-  cluster_arrive();  // no remote reads after this point
   const int eq_incl = warp_incl_scan(eqq);
   const int sel_q = gq + max(0, min(eqq, take_eq - (eq_incl - eqq)));
   int sel_before = sel_q;
@@ -599,6 +668,11 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
   const int s_in = warp_incl_scan(s_l);
   int eq_seen = eq_before + __shfl_sync(0xffffffffu, e_ex, warp);
   int pos = sel_before + __shfl_sync(0xffffffffu, s_in - s_l, warp);
+  if (failed) {  // (warp-uniform) values received may be incomplete: write no ids
+    if (lane == 0) record_error(c.status, RESA_DEV_WAIT_TIMEOUT, b * c.Hkv + h);
+    asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+    return;
+  }
   for (int i0 = w0; i0 < w1; i0 += 32) {
     const int i = i0 + lane;
     bool is_gt, is_eq;
@@ -611,9 +685,8 @@ __global__ void __launch_bounds__(kTopnThreads) topn_kernel(CacheView c, const f
     eq_seen += __popc(eqm);
     pos += __popc(selm);
   }
-  for (int i = n + rank * kTopnThreads + tid; i < n_cap; i += kTopnCluster * kTopnThreads) out[i] = -1;
+  for (int i = n + static_cast<int>(rank) * kTopnThreads + tid; i < n_cap; i += kTopnCluster * kTopnThreads) out[i] = -1;
   if (rank == 0 && tid == 0) counts[b * c.Hkv + h] = n;
-  cluster_wait();  // no CTA leaves while a peer may still read its shared memory
 }
 
 // One-CTA radix select, grid (KV head, sequence), for caches of up to
@@ -801,13 +874,15 @@ int select_max_blocks() { return kTopnCluster * (kTopnSmemMax / static_cast<int>
 cudaError_t launch_select(const CacheView& c, const uint16_t* q, double keep, int n_min, int n_local,
                           int32_t* indices, int32_t* counts, int n_cap, float* scores, int sm_count,
                           cudaStream_t st) {
-  cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(score_kernel), kScoreSmem, 3);
+  cudaError_t e =
+      ensure_smem_attr(reinterpret_cast<const void*>(score_kernel), kScoreSmem + score_table_bytes(kMaxBatch), 3);
   if (e != cudaSuccess) return e;
   // one persistent CTA per SM (never more than the pieces there can be)
   const long long max_pieces =
       static_cast<long long>(c.B) * c.Hkv * ((c.max_blocks + kPieceBlocks - 1) / kPieceBlocks);
   const int grid = static_cast<int>(max(1LL, min(static_cast<long long>(sm_count), max_pieces)));
-  e = launch_pdl(score_kernel, dim3(grid), dim3(kScoreWarps * 32), kScoreSmem, st, c, q, scores);
+  e = launch_pdl(score_kernel, dim3(grid), dim3(kScoreWarps * 32), kScoreSmem + score_table_bytes(c.B), st, c, q,
+                 scores);
   if (e != cudaSuccess) return e;
   const size_t smem = select_smem_bytes(c.max_blocks);
   if (c.max_blocks <= kTopnCtaMaxBlocks)
