@@ -202,6 +202,43 @@ def test_select_ties_go_to_lower_index(maxb):
     assert idx[0, 0, :4].tolist() == [0, 1, 2, 39]
 
 
+def _tied_unit(M, tied, scale, seed):
+    """Keys of one KV head: M random blocks, with the blocks `tied` replaced
+    by one shared block scaled by `scale` (identical summaries, so identical
+    scores in the oracle and on the GPU)."""
+    K = synth.normal_bf16(synth.rng(seed), (1, M * 16, 128))
+    blk = synth.normal_bf16(synth.rng(seed + 1), (1, 16, 128), scale)
+    for m in tied:
+        K[:, m * 16:(m + 1) * 16] = blk
+    V = synth.normal_bf16(synth.rng(seed + 2), (1, M * 16, 128))
+    return K, V
+
+
+@pytest.mark.parametrize("tied,scale,keep", [
+    (range(700, 1300), 4.0, 0.04),   # 600 top-scoring equal blocks over two CTAs: the boundary bucket is gathered
+    (range(0, 6397), 1.0, 0.1),      # ~6,400 equal blocks at the boundary: exchanged passes and counts
+])
+def test_select_cluster_ties_at_the_boundary(tied, scale, keep):
+    """Cluster top-n (6,400 blocks, 800 per CTA) with the n-th largest score
+    shared by many blocks: the ids equal the oracle's exactly, ties to the
+    lower ids across CTAs."""
+    M, g = 6400, 4
+    K, V = _tied_unit(M, tied, scale, 91)
+    maxb = M + 10
+    cache = H.make_cache([K], [V], g, maxb, compact=True)
+    q = synth.normal_bf16(synth.rng(95), (1, g, 128))
+    p = resa.params(keep, 0, 1)
+    n_cap = resa.resa_max_selected(cache.struct, p)
+    idx, cnt = run_select(cache, q, p, n_cap)
+    assert resa.resa_read_device_error(cache.struct) == (0, 0)
+    st = H.oracle_state(K, V, maxb * 16)
+    _, scores, n = O.select_for_group(st, 0, O.widen_bf16(q[0]), O.ResaParams(keep, 0, 1))
+    assert cnt[0, 0] == n
+    tie = scores[tied[0]]
+    assert np.sum(scores > tie) < n - 1 < np.sum(scores >= tie)  # the boundary lies inside the tied blocks
+    assert np.array_equal(idx[0, 0, :n], O.select_blocks(scores, n, 1))
+
+
 @pytest.mark.parametrize("maxb", [110, 6200])  # one-CTA and cluster top-n
 def test_select_budget_over_cap_is_reported_and_clamped(maxb):
     Ks, Vs = seq_inputs(9, 1, 1, [1600])
