@@ -140,7 +140,9 @@ resa_status_t resa_max_selected(const resa_cache_t* cache, const resa_params_t* 
 /*
  * Number of key splits resa_sparse_decode uses when num_splits == 0, for the
  * current device: Algorithm 2's num_splits, chosen so that
- * batch * num_kv_heads * splits fills the SMs (Section 2.4).
+ * batch * num_kv_heads * splits fills the SMs in one wave (Section 2.4), with
+ * one resident CTA per SM instead of two when two would leave a split fewer
+ * than 16 of the n_cap selected blocks, and at least two blocks per split.
  */
 resa_status_t resa_decode_num_splits(const resa_cache_t* cache, int32_t n_cap, int32_t* splits_out);
 

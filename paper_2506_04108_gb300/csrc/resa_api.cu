@@ -166,9 +166,14 @@ resa_status_t auto_decode_splits(const resa_cache_t* c, int n_cap, int* out) {
   if (s != RESA_OK) return s;
   // Algorithm 2's num_splits: as many splits as fit in one wave of resident
   // decode CTAs over batch * KV heads (no tail wave), with at least two
-  // selected blocks per split.
+  // selected blocks per split. Fewer CTAs per SM are resident when the full
+  // count would leave a split fewer than 16 selected blocks (measured: batch
+  // 1 at 256K, 4 units of 820 blocks, runs its decode step faster with 38
+  // splits of ~22 blocks than with 76 of ~11).
   const int units = c->batch * c->num_kv_heads;
-  int splits = sms * decode_ctas_per_sm() / units;
+  int per_sm = decode_ctas_per_sm();
+  while (per_sm > 1 && n_cap < 16 * (sms * per_sm / units)) --per_sm;
+  int splits = sms * per_sm / units;
   const int max_by_blocks = n_cap / 2 > 1 ? n_cap / 2 : 1;
   if (splits > max_by_blocks) splits = max_by_blocks;
   if (splits > 256) splits = 256;
