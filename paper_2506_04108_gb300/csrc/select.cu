@@ -15,18 +15,18 @@
 //               order-preserving keys of the other blocks, found by a radix
 //               select over key - min key with 8-bit digits from the top
 //               significant bit of the unit's key range (keys staged in shared
-//               memory; in the cluster form the histograms are summed across
-//               the cluster through distributed shared memory). The selected
+//               memory; in the cluster form every exchange between the CTAs,
+//               extremes, histograms and counts, is stored into the other
+//               CTAs' shared memory by stores that complete on the
+//               receiver's mbarrier). The selected
 //               ids are written in ascending order by a ballot compaction that
 //               resolves ties at the threshold toward the lower block index.
 //
 // Both top-n kernels read the length and evaluate Eq. 5 before waiting on the
 // score kernel: that kernel lets its dependents launch only after its own wait
-// on the preceding kernel (the append commit that advances the length) has
-// returned, and the length is read from L2.
-#include <cooperative_groups.h>
-
-#include <atomic>
+// on the preceding kernel (the append commit, or the previous fused step's
+// merge, that advances the length) has returned, and the length is read from
+// L2.
 
 #include "resa_device.cuh"
 #include "resa_launch.h"
