@@ -354,10 +354,11 @@ def oracle_period(sample: dict) -> float:
     return time.perf_counter() - t0
 
 
-def run_oracle_subprocess(sample: dict, threads: int = 1, repeats: int = 1):
-    """Time oracle_period `repeats` times in a fresh process whose BLAS/OpenMP
-    pools are pinned to `threads` (so `cores` is what the oracle actually
-    used); returns the list of per-repeat seconds."""
+def run_oracle_subprocess(sample: dict, threads: int = 1, repeats: int = 1, min_seconds: float = 0.0):
+    """Time oracle_period `repeats` times, then more until `min_seconds` of
+    work have been timed (at most ORACLE_MAX_REPEATS periods), in a fresh
+    process whose BLAS/OpenMP pools are pinned to `threads` (so `cores` is
+    what the oracle actually used); returns the list of per-repeat seconds."""
     with tempfile.TemporaryDirectory() as d:
         path = os.path.join(d, "sample.npz")
         np.savez(path, **sample)
@@ -365,7 +366,8 @@ def run_oracle_subprocess(sample: dict, threads: int = 1, repeats: int = 1):
         for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "BLIS_NUM_THREADS"):
             env[v] = str(threads)
         r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-worker", path,
-                            "--repeats", str(repeats)], env=env, capture_output=True, text=True, timeout=3600)
+                            "--repeats", str(repeats), "--min-seconds", str(min_seconds)],
+                           env=env, capture_output=True, text=True, timeout=3600)
         if r.returncode != 0:
             raise RuntimeError(f"oracle worker failed: {r.stderr[-2000:]}")
         return json.loads(r.stdout.strip().splitlines()[-1])["seconds"]
@@ -581,10 +583,12 @@ def run_ours(args, w: synth.Workload):
                   "v": bits(layers[0].v[:, 0]), "rq": bits(layers[0].rq[0]), "rk": bits(layers[0].rk[0]),
                   "rv": bits(layers[0].rv[0]), "f": f, "keep": w.keep, "n_min": w.n_min_blocks,
                   "n_local": w.n_local_blocks}
-        secs_cpu = run_oracle_subprocess(sample, threads=1)[0]
-        cpu = {"value": round(f / secs_cpu, 2), "unit": UNIT, "cores": 1, "kind": "oracle",
+        times = run_oracle_subprocess(sample, threads=1, min_seconds=CPU_BASELINE_SECONDS)
+        secs_cpu = sum(times)
+        cpu = {"value": round(f * len(times) / secs_cpu, 2), "unit": UNIT, "cores": 1, "kind": "oracle",
                "sample": f"1 of {B} sequences x 1 of {L} layers: {f} decode steps + 1 rectification at context "
-                         f"{w.context} (fp64 numpy, 1 BLAS thread)", "seconds": round(secs_cpu, 3)}
+                         f"{w.context}, timed {len(times)} times (fp64 numpy, 1 BLAS thread)",
+               "seconds": round(secs_cpu, 3)}
 
     launches = args.steps * L * (f * LayerCache.KERNELS_PER_DECODE_STEP + LayerCache.KERNELS_PER_RECTIFY)
     line = {"metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -601,6 +605,8 @@ def run_ours(args, w: synth.Workload):
 
 
 ATTR_REPS = 3
+CPU_BASELINE_SECONDS = 10.0  # oracle work timed for cpu_baseline (whole periods, at least one)
+ORACLE_MAX_REPEATS = 400
 TOPN_CTA_MAX_BLOCKS = 6144  # caches of up to this many blocks per sequence use the one-CTA top-n
 
 
@@ -914,10 +920,14 @@ def main():
                     help="time rectification over the 16K/64K/256K x f 16/32/64 grid instead")
     ap.add_argument("--oracle-worker", default=None, help=argparse.SUPPRESS)
     ap.add_argument("--repeats", type=int, default=1, help=argparse.SUPPRESS)
+    ap.add_argument("--min-seconds", type=float, default=0.0, help=argparse.SUPPRESS)
     args = ap.parse_args()
     if args.oracle_worker:
         sample = dict(np.load(args.oracle_worker))
-        print(json.dumps({"seconds": [oracle_period(sample) for _ in range(args.repeats)]}))
+        secs = [oracle_period(sample) for _ in range(args.repeats)]
+        while sum(secs) < args.min_seconds and len(secs) < ORACLE_MAX_REPEATS:
+            secs.append(oracle_period(sample))
+        print(json.dumps({"seconds": secs}))
         return
     if args.warmup < 3 and args.impl == "ours":
         ap.error("--warmup must be >= 3")
