@@ -1,5 +1,6 @@
 """Host-side logic of bench.py (CPU only): the algorithmic byte model against
-Eq. 6, and the multi-rank aggregation over a world_size-2 gloo group."""
+Eq. 6, the multi-rank aggregation over a world_size-2 gloo group, and the
+timing loop of the CPU baseline."""
 import math
 import os
 
@@ -9,6 +10,7 @@ import torch.distributed as dist
 import torch.multiprocessing as mp
 
 import bench
+from paper_2506_04108_gb300 import synth
 
 
 def test_step_bytes_follow_eq6():
@@ -68,3 +70,14 @@ def test_two_rank_gloo_aggregation():
 def test_single_process_helpers_are_identity():
     assert bench.max_over_ranks(3.5) == 3.5
     assert bench.aggregate(10.0, 2.0, 1) == 5.0
+
+
+def test_oracle_worker_times_whole_periods_until_min_seconds():
+    """cpu_baseline's timing loop: at least the requested periods, then more
+    until the timed work reaches min_seconds (a small 4K-shaped sample)."""
+    w = synth.WORKLOADS["b1_h8kv2_ctx4k_f8"]
+    s = bench.host_sample(w, 512)
+    times = bench.run_oracle_subprocess(s, threads=1, repeats=2, min_seconds=0.5)
+    assert len(times) >= 2 and all(t > 0 for t in times)
+    assert sum(times) >= 0.5 or len(times) == bench.ORACLE_MAX_REPEATS
+    assert sum(times[:-1]) < 0.5 or len(times) == 2  # stops at the first period past the bound
