@@ -1,9 +1,10 @@
 // Block selection (Section 2.1 "Block Selection"; Eq. 4 and Eq. 5).
 //
 // score_kernel  persistent, one CTA per SM: each of its 16 warps streams 6 KB
-//               pieces of the block summaries with its own bulk copies through
-//               its own shared-memory ring and scores them with the pooled
-//               query of the piece's GQA group (mean of the g heads, fp32); a
+//               (small caches: 4 KB) pieces of the block summaries with its
+//               own bulk copies through its own shared-memory ring and
+//               scores them with the pooled query of the piece's GQA group
+//               (mean of the g heads, fp32); a
 //               half-warp takes one block, a lane one 16-byte piece (8 dims)
 //               of k_min and k_max, and the 128-dim sum is a fixed-order
 //               butterfly over the 16 lanes.
@@ -69,26 +70,38 @@ __device__ __forceinline__ float quest_term8(const float* qa, const uint32_t* sg
 }
 
 // Persistent score kernel: one CTA per SM. The (sequence, KV head) units'
-// summaries are cut into pieces of 12 blocks (6 KB, contiguous); CTA x owns
-// the piece range [x * per, (x + 1) * per) of the flattened piece list and
-// its warp w takes every 16th piece of it (w, w + 16, ...). Each warp streams
-// its pieces with 1-D bulk copies issued by its own lane 0 through its own
-// 2-stage shared-memory ring: copies issued by one thread complete one after
-// another, so sixteen independent issuers keep enough bytes in flight per SM
-// (measured: 6 KB pieces in 2 stages beat 4 KB in 3 and 8 KB with 12 warps).
-// A half-warp scores one block, a lane one 16-byte piece (8 dims) of k_min
-// and k_max, and the 128-dim sum ends in a fixed-order 16-lane butterfly.
+// summaries are cut into pieces of kPieceBlocks blocks (contiguous); CTA x
+// owns the piece range [x * per, (x + 1) * per) of the flattened piece list
+// and its warp w takes every 16th piece of it (w, w + 16, ...). Each warp
+// streams its pieces with 1-D bulk copies issued by its own lane 0 through
+// its own kScoreStages-stage shared-memory ring: copies issued by one thread
+// complete one after another, so sixteen independent issuers keep enough
+// bytes in flight per SM. Two shapes, the same 192 KB of rings: 12-block
+// (6 KB) pieces in 2 stages when the cache has at least one such piece per
+// warp of the grid (measured: they beat 8 blocks in 3 stages, and 16 blocks
+// with 12 warps, at 32K x 8 and 256K x 1), else 8-block (4 KB) pieces in 3
+// stages, which give more warps a piece. A half-warp scores one block, a
+// lane one 16-byte piece (8 dims) of k_min and k_max, and the 128-dim sum
+// ends in a fixed-order 16-lane butterfly.
 constexpr int kScoreWarps = 16;
-constexpr int kScoreStages = 2;                                    // pieces in flight per warp
 constexpr int kMaxBatch = 1024;  // sequences per call supported by the score kernel
-constexpr int kPieceBlocks = 12;
-constexpr int kPieceBytes = kPieceBlocks * 2 * kHeadDim * 2;       // 6 KB
-constexpr int kScoreRing = kScoreWarps * kScoreStages * kPieceBytes;  // 192 KB
-constexpr int kScoreSmem = kScoreRing + kScoreWarps * kScoreStages * 8;  // + score_table_bytes(B)
+constexpr int score_piece_bytes(int piece_blocks) { return piece_blocks * 2 * kHeadDim * 2; }
+constexpr int score_ring_bytes(int piece_blocks, int stages) {
+  return kScoreWarps * stages * score_piece_bytes(piece_blocks);
+}
+// rings and their barriers; the per-sequence tables (score_table_bytes) follow
+constexpr int score_smem_bytes(int piece_blocks, int stages) {
+  return score_ring_bytes(piece_blocks, stages) + kScoreWarps * stages * 8;
+}
 constexpr int score_table_bytes(int B) { return (3 * B + 1) * static_cast<int>(sizeof(int)); }
 
+template <int kPieceBlocks, int kScoreStages>
 __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c, const uint16_t* __restrict__ q,
                                                                     float* __restrict__ scores) {
+  static_assert(kPieceBlocks % 2 == 0, "two half-warps score a piece's blocks in pairs");
+  constexpr int kPieceBytes = score_piece_bytes(kPieceBlocks);
+  constexpr int kScoreRing = score_ring_bytes(kPieceBlocks, kScoreStages);
+  constexpr int kScoreSmem = score_smem_bytes(kPieceBlocks, kScoreStages);
   extern __shared__ __align__(1024) uint8_t smem[];
   // per-sequence block counts and the piece prefix over (sequence, head)
   // units, after the rings and their barriers (sized by the batch, so that
@@ -871,18 +884,29 @@ size_t select_smem_bytes(int max_blocks) {
 
 int select_max_blocks() { return kTopnCluster * (kTopnSmemMax / static_cast<int>(sizeof(uint32_t))); }
 
-cudaError_t launch_select(const CacheView& c, const uint16_t* q, double keep, int n_min, int n_local,
-                          int32_t* indices, int32_t* counts, int n_cap, float* scores, int sm_count,
-                          cudaStream_t st) {
+template <int kPieceBlocks, int kScoreStages>
+cudaError_t launch_score(const CacheView& c, const uint16_t* q, float* scores, int sm_count, cudaStream_t st,
+                         int attr_slot) {
+  constexpr int kSmem = score_smem_bytes(kPieceBlocks, kScoreStages);
+  const auto kernel = score_kernel<kPieceBlocks, kScoreStages>;
   cudaError_t e =
-      ensure_smem_attr(reinterpret_cast<const void*>(score_kernel), kScoreSmem + score_table_bytes(kMaxBatch), 3);
+      ensure_smem_attr(reinterpret_cast<const void*>(kernel), kSmem + score_table_bytes(kMaxBatch), attr_slot);
   if (e != cudaSuccess) return e;
   // one persistent CTA per SM (never more than the pieces there can be)
   const long long max_pieces =
       static_cast<long long>(c.B) * c.Hkv * ((c.max_blocks + kPieceBlocks - 1) / kPieceBlocks);
   const int grid = static_cast<int>(max(1LL, min(static_cast<long long>(sm_count), max_pieces)));
-  e = launch_pdl(score_kernel, dim3(grid), dim3(kScoreWarps * 32), kScoreSmem + score_table_bytes(c.B), st, c, q,
-                 scores);
+  return launch_pdl(kernel, dim3(grid), dim3(kScoreWarps * 32), kSmem + score_table_bytes(c.B), st, c, q, scores);
+}
+
+cudaError_t launch_select(const CacheView& c, const uint16_t* q, double keep, int n_min, int n_local,
+                          int32_t* indices, int32_t* counts, int n_cap, float* scores, int sm_count,
+                          cudaStream_t st) {
+  // 6 KB pieces when there is at least one per warp of a full grid
+  const long long pieces12 = static_cast<long long>(c.B) * c.Hkv * ((c.max_blocks + 11) / 12);
+  cudaError_t e = pieces12 >= static_cast<long long>(sm_count) * kScoreWarps
+                      ? launch_score<12, 2>(c, q, scores, sm_count, st, 3)
+                      : launch_score<8, 3>(c, q, scores, sm_count, st, 4);
   if (e != cudaSuccess) return e;
   const size_t smem = select_smem_bytes(c.max_blocks);
   if (c.max_blocks <= kTopnCtaMaxBlocks)
