@@ -270,6 +270,27 @@ class LayerCache:
         self.rv = dv.transpose(0, 1).contiguous()
         self.out = torch.empty((f, B, Hq, HEAD_DIM), dtype=torch.bfloat16, device=device)
         self.rout = torch.empty((B, f, Hq, HEAD_DIM), dtype=torch.bfloat16, device=device)
+        self.needle_target = None
+        if w.needle_blocks > 0:
+            # Needle workload: per (sequence, KV head) a seeded set of needle
+            # blocks of the prompt; at each step every query head of the group
+            # is q = z + 2 k*, k* a random key of a random needle block (the
+            # recipe of synth.decode_inputs, drawn here on the device pools).
+            gn = synth.rng(seed * 7 + 3)
+            g, nb = w.group, w.needle_blocks
+            needles = np.stack([np.stack([gn.choice(w.context // BLOCK, size=nb, replace=False)
+                                          for _ in range(Hkv)]) for _ in range(B)])          # [B, Hkv, nb]
+            pick = gn.integers(nb, size=(f, B, Hkv))
+            row = gn.integers(BLOCK, size=(f, B, Hkv))
+            blk = np.take_along_axis(np.broadcast_to(needles, (f, B, Hkv, nb)), pick[..., None], axis=3)[..., 0]
+            page = pt[np.arange(B)[None, :, None], blk]
+            heads = np.broadcast_to(np.arange(Hkv)[None, None, :], blk.shape)
+            kstar = self.cache.k_pool[torch.from_numpy(page).long().to(device),
+                                      torch.from_numpy(np.ascontiguousarray(heads)).long().to(device),
+                                      torch.from_numpy(row).long().to(device)].float()       # [f, B, Hkv, d]
+            z = torch.randn((f, B, Hkv, g, HEAD_DIM), generator=tg, device=device)
+            self.q = (z + 2.0 * kstar[:, :, :, None, :]).reshape(f, B, Hq, HEAD_DIM).to(torch.bfloat16)
+            self.needle_target = torch.from_numpy(blk.astype(np.int32)).to(device)              # [f, B, Hkv]
 
     # kernels per call: the fused decode step 4 (score, top-n, decode, merge),
     # rectify 2, overwrite 1
@@ -304,6 +325,24 @@ class LayerCache:
         """Rectification branch of Algorithm 1 for this layer."""
         self.rectify_attention()
         self.overwrite()
+
+
+def needle_recall(layers) -> dict:
+    """Informational: the fraction of (step, sequence, KV head) where the
+    needle block the query was built from is among the selected blocks, over
+    one eager period of fused decode steps on every layer (not timed)."""
+    import torch
+    f = layers[0].w.f
+    hits = torch.zeros((), dtype=torch.int64, device=layers[0].idx.device)
+    n = 0
+    for t in range(f):
+        for Lc in layers:
+            Lc.decode(t)
+            hits += (Lc.idx == Lc.needle_target[t][..., None]).any(dim=-1).sum()
+            n += Lc.needle_target[t].numel()
+    check_device_errors(layers)
+    return {"value": round(int(hits.item()) / n, 4), "samples": n, "informational": True,
+            "what": "needle block of the step's query selected (Eq. 4/5), one period on every layer"}
 
 
 def run_period(layers):
@@ -449,6 +488,57 @@ def check_device_errors(layers):
             raise RuntimeError(f"device error {resa.DEVICE_ERRORS.get(code)} detail {detail}")
 
 
+# The step is decode_step (f x L), rectify and overwrite (L each); select,
+# decode and commit are the pieces decode_step fuses, timed as their own calls
+# for the per-kernel rooflines. decode_step and commit append f tokens per
+# replay of their graph.
+IN_STEP = ("decode_step", "rectify", "overwrite")
+APPENDING_KINDS = ("decode_step", "commit")
+
+
+def time_call_kinds(layers, device):
+    """Mean microseconds per call of each call type: one CUDA graph per type
+    holding the period's calls of that type in step order (f x L or L calls),
+    one warm replay, then ATTR_REPS replays timed with CUDA events. The two
+    appending types advance every sequence by f * (1 + ATTR_REPS) tokens."""
+    f, L = layers[0].w.f, len(layers)
+    kinds = {
+        "decode_step": lambda: [Lc.decode(t) for t in range(f) for Lc in layers],
+        "select": lambda: [Lc.select(t) for t in range(f) for Lc in layers],
+        "decode": lambda: [Lc.sparse_decode(t) for t in range(f) for Lc in layers],
+        "rectify": lambda: [Lc.rectify_attention() for Lc in layers],
+        "overwrite": lambda: [Lc.overwrite() for Lc in layers],
+        "commit": lambda: [Lc.commit(t) for t in range(f) for Lc in layers],
+    }
+    ncalls = {"decode_step": f * L, "select": f * L, "decode": f * L, "rectify": L, "overwrite": L, "commit": f * L}
+    mean_us = {}
+    for kind, fn in kinds.items():
+        gk = capture(fn, device)             # capture does not execute
+        gk.replay()                          # warm
+        mean_us[kind] = time_graph(gk, ATTR_REPS) / ncalls[kind] * 1e6
+        del gk
+    check_device_errors(layers)
+    return mean_us, ncalls
+
+
+def call_bytes(w: synth.Workload, T: int) -> dict:
+    """Algorithmic bytes of one call of each type at context T (select at the
+    middle of the appending replays' range)."""
+    B, f = w.batch, w.f
+    Tm = T + f // 2
+    return {
+        "decode_step": (commit_bytes(B, w.num_kv_heads, 1) +
+                        select_bytes(B, w.num_q_heads, w.num_kv_heads, Tm, w.keep, w.n_min_blocks, w.n_local_blocks) +
+                        decode_bytes(B, w.num_q_heads, w.num_kv_heads, T, w.keep, w.n_min_blocks,
+                                     w.n_local_blocks)),
+        "commit": commit_bytes(B, w.num_kv_heads, 1),
+        "select": select_bytes(B, w.num_q_heads, w.num_kv_heads, Tm, w.keep, w.n_min_blocks, w.n_local_blocks),
+        "decode": decode_bytes(B, w.num_q_heads, w.num_kv_heads, T, w.keep, w.n_min_blocks, w.n_local_blocks),
+        "rectify": rectify_bytes(B, w.num_q_heads, w.num_kv_heads, T, f),
+        "overwrite": commit_bytes(B, w.num_kv_heads, f),
+    }
+
+
 def run_ours(args, w: synth.Workload):
     import torch
     rank, world, local = dist_env()
@@ -463,7 +553,7 @@ def run_ours(args, w: synth.Workload):
 
     L, f, B = args.layers, w.f, w.batch
     # periods that append f tokens: warm-up call, graph warm-up/timed/e2e replays, attribution commits
-    periods_total = 1 + args.warmup + args.steps + (1 + args.steps) + 2 * (1 + ATTR_REPS)
+    periods_total = 1 + args.warmup + args.steps + (1 + args.steps) + 2 * (1 + ATTR_REPS) + 1
     capacity = ((w.context + f * periods_total + BLOCK) // BLOCK + 1) * BLOCK
     layers = [LayerCache(w, capacity, w.seed * 100 + 17 * rank + i, device) for i in range(L)]
     torch.cuda.synchronize()
@@ -503,45 +593,11 @@ def run_ours(args, w: synth.Workload):
     T += f * (args.steps + 1)  # the timed steps and the warm replay of the second buffer set's graph
 
     # ---- per-call durations: one graph per call type, the period's calls of that type in order ----
-    # The step is decode_step (f x L), rectify and overwrite (L each); select,
-    # decode and commit are the pieces decode_step fuses, timed as their own
-    # calls for the per-kernel rooflines.
     T_attr = T
-    appends = ("decode_step", "commit")
-    kinds = {
-        "decode_step": lambda: [Lc.decode(t) for t in range(f) for Lc in layers],
-        "select": lambda: [Lc.select(t) for t in range(f) for Lc in layers],
-        "decode": lambda: [Lc.sparse_decode(t) for t in range(f) for Lc in layers],
-        "rectify": lambda: [Lc.rectify_attention() for Lc in layers],
-        "overwrite": lambda: [Lc.overwrite() for Lc in layers],
-        "commit": lambda: [Lc.commit(t) for t in range(f) for Lc in layers],
-    }
-    ncalls = {"decode_step": f * L, "select": f * L, "decode": f * L, "rectify": L, "overwrite": L, "commit": f * L}
-    in_step = ("decode_step", "rectify", "overwrite")
-    mean_us = {}
-    for kind, fn in kinds.items():
-        gk = capture(fn, device)             # capture does not execute
-        gk.replay()                          # warm
-        if kind in appends:
-            T += f
-        mean_us[kind] = time_graph(gk, ATTR_REPS) / ncalls[kind] * 1e6
-        if kind in appends:
-            T += f * ATTR_REPS
-        del gk
-    check_device_errors(layers)
-    Tm = T_attr + f // 2
-    algo = {
-        "decode_step": (commit_bytes(B, w.num_kv_heads, 1) +
-                        select_bytes(B, w.num_q_heads, w.num_kv_heads, Tm, w.keep, w.n_min_blocks, w.n_local_blocks) +
-                        decode_bytes(B, w.num_q_heads, w.num_kv_heads, T_attr, w.keep, w.n_min_blocks,
-                                     w.n_local_blocks)),
-        "commit": commit_bytes(B, w.num_kv_heads, 1),
-        "select": select_bytes(B, w.num_q_heads, w.num_kv_heads, Tm, w.keep, w.n_min_blocks, w.n_local_blocks),
-        "decode": decode_bytes(B, w.num_q_heads, w.num_kv_heads, T_attr, w.keep, w.n_min_blocks,
-                               w.n_local_blocks),
-        "rectify": rectify_bytes(B, w.num_q_heads, w.num_kv_heads, T_attr, f),
-        "overwrite": commit_bytes(B, w.num_kv_heads, f),
-    }
+    mean_us, ncalls = time_call_kinds(layers, device)
+    T += f * 2 * (1 + ATTR_REPS)
+    in_step = IN_STEP
+    algo = call_bytes(w, T_attr)
     peaks, peak_kind = load_peaks()
     hbm = float(peaks["hbm_gbs"])
     per_step_us = {k: mean_us[k] * ncalls[k] for k in mean_us}
@@ -576,6 +632,11 @@ def run_ours(args, w: synth.Workload):
                 "algorithmic_bytes_per_launch": int(algo[dominant]),
                 "timing": "CUDA events around a graph of the step's calls of this kind; per call = total / calls"}
 
+    recall = needle_recall(layers) if w.needle_blocks > 0 else None
+    targets = None
+    if world == 1 and not args.no_targets:
+        targets = run_targets(device)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         Kb, Vb = host_logical_kv(layers[0].cache, 0, w.context)
@@ -596,7 +657,9 @@ def run_ours(args, w: synth.Workload):
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": config_of(w, args), "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": launches, "clocks": clk, "calls": calls, "context_at_timed_start": T_timed0,
-            "eq6_ratio": round(eq6_ratio(BLOCK, w.keep, f), 5)}
+            "eq6_ratio": round(eq6_ratio(BLOCK, w.keep, f), 5), "targets": targets}
+    if recall is not None:
+        line["needle_recall"] = recall
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -692,12 +755,77 @@ def run_e2e(args, layers, graph):
                     "buffer sets so step i + 1's inputs and step i - 1's outputs cross while step i computes"}
 
 
+def rectify_cell(T: int, f: int, device, peaks: dict, peak_kind: str) -> dict:
+    """One cell of the rectification sweep: dense causal attention of f new
+    queries (28 q / 4 KV heads, d 128, batch 1) against a cached context T,
+    then the K/V overwrite and block-summary refresh of the touched blocks.
+    Enough independent caches rotate that the rotation's working set exceeds
+    L2; each call is timed from a CUDA graph of the rotation with CUDA events."""
+    import torch
+    from paper_2506_04108_gb300 import resa
+    Hq, Hkv, B = 28, 4, 1
+    ncache = max(1, math.ceil(300e6 / (B * Hkv * T * 512)))
+    caches = []
+    for i in range(ncache):
+        maxb = (T + BLOCK - 1) // BLOCK + 1
+        pt = synth.page_table(synth.rng(synth.RECTIFY_SWEEP_SEED + i), B, maxb)
+        cch = resa.PagedKVCache(B, Hq, Hkv, maxb, pt, device=device, zero_pools=False)
+        tg = torch.Generator(device=device)
+        tg.manual_seed(synth.RECTIFY_SWEEP_SEED * 10 + i)
+        for pool in (cch.k_pool, cch.v_pool):
+            pool.copy_(torch.randn(pool.shape, generator=tg, device=device))
+        cch.seq_lens.fill_(T)
+        resa.resa_update_summaries(cch.struct, 0, -1)
+        qn = torch.randn((B, f, Hq, HEAD_DIM), generator=tg, device=device).to(torch.bfloat16)
+        kn = torch.randn((B, f, Hkv, HEAD_DIM), generator=tg, device=device).to(torch.bfloat16)
+        vn = torch.randn((B, f, Hkv, HEAD_DIM), generator=tg, device=device).to(torch.bfloat16)
+        out = torch.empty_like(qn)
+        nb = resa.resa_workspace_size(cch.struct, 8, 0, f)
+        ws = torch.empty(nb, dtype=torch.uint8, device=device)
+        caches.append((cch, qn, kn, vn, out, ws, nb))
+    p = resa.params(0.1, 0, 0)
+
+    def one(c):
+        cch, qn, kn, vn, out, ws, nb = c
+        resa.resa_rectify_attention(cch.struct, qn, kn, vn, f, p, out, None, ws, nb)
+        resa.resa_commit_kv(cch.struct, kn, vn, f, True)
+
+    def rect_only(c):
+        cch, qn, kn, vn, out, ws, nb = c
+        resa.resa_rectify_attention(cch.struct, qn, kn, vn, f, p, out, None, ws, nb)
+    for c in caches:
+        one(c)
+    torch.cuda.synchronize()
+    reps = max(2, math.ceil(8 / ncache))
+    g_all = capture(lambda: [one(c) for _ in range(reps) for c in caches], device)
+    g_rect = capture(lambda: [rect_only(c) for _ in range(reps) for c in caches], device)
+    g_all.replay()
+    g_rect.replay()
+    calls = reps * ncache
+    t_all = time_graph(g_all, 3) / calls
+    t_rect = time_graph(g_rect, 3) / calls
+    for c in caches:
+        code, _ = resa.resa_read_device_error(c[0].struct)
+        if code:
+            raise RuntimeError(f"device error {resa.DEVICE_ERRORS.get(code)}")
+    flops = rectify_flops(B, Hq, T, f)
+    byts = rectify_bytes(B, Hq, Hkv, T, f)
+    tf = flops / t_rect / 1e12
+    gbs = byts / t_rect / 1e9
+    del caches, g_all, g_rect
+    torch.cuda.empty_cache()
+    return {"context": T, "f": f, "batch": B, "caches_rotated": ncache,
+            "rectify_us": round(t_rect * 1e6, 2), "rectify_plus_overwrite_us": round(t_all * 1e6, 2),
+            "TFLOP/s": round(tf, 1), "frac_bf16_burst": round(tf / float(peaks["bf16_tflops"]), 3),
+            "frac_bf16_sustained": round(tf / float(peaks["bf16_tflops_sustained"]), 3),
+            "GB/s": round(gbs, 1), "frac_hbm": round(gbs / float(peaks["hbm_gbs"]), 3),
+            "bound": "hbm" if 7 * f < float(peaks["bf16_tflops"]) / float(peaks["hbm_gbs"]) * 1e3 else "tensor",
+            "peak_kind": peak_kind}
+
+
 def run_rectify_sweep(args):
-    """Rectification-only sweep (the f x context grid): per cell, dense causal
-    attention of f new queries (28 q / 4 KV heads, d 128, batch 1) against a
-    cached context T, then the K/V overwrite and block-summary refresh of the
-    touched blocks. Enough independent caches rotate per cell that the
-    rotation's working set exceeds L2. One JSON line per cell."""
+    """Rectification-only sweep (the f x context grid of synth.RECTIFY_SWEEP),
+    one JSON line per cell (see rectify_cell)."""
     import torch
     from paper_2506_04108_gb300 import build as _b
     from paper_2506_04108_gb300 import resa
@@ -706,66 +834,68 @@ def run_rectify_sweep(args):
     device = torch.device("cuda", 0)
     torch.cuda.set_device(0)
     peaks, peak_kind = load_peaks()
-    Hq, Hkv, B = 28, 4, 1
     for T, f in synth.RECTIFY_SWEEP:
-        ncache = max(1, math.ceil(300e6 / (B * Hkv * T * 512)))
-        caches = []
-        for i in range(ncache):
-            maxb = (T + BLOCK - 1) // BLOCK + 1
-            pt = synth.page_table(synth.rng(synth.RECTIFY_SWEEP_SEED + i), B, maxb)
-            cch = resa.PagedKVCache(B, Hq, Hkv, maxb, pt, device=device, zero_pools=False)
-            tg = torch.Generator(device=device)
-            tg.manual_seed(synth.RECTIFY_SWEEP_SEED * 10 + i)
-            for pool in (cch.k_pool, cch.v_pool):
-                pool.copy_(torch.randn(pool.shape, generator=tg, device=device))
-            cch.seq_lens.fill_(T)
-            resa.resa_update_summaries(cch.struct, 0, -1)
-            qn = torch.randn((B, f, Hq, HEAD_DIM), generator=tg, device=device).to(torch.bfloat16)
-            kn = torch.randn((B, f, Hkv, HEAD_DIM), generator=tg, device=device).to(torch.bfloat16)
-            vn = torch.randn((B, f, Hkv, HEAD_DIM), generator=tg, device=device).to(torch.bfloat16)
-            out = torch.empty_like(qn)
-            nb = resa.resa_workspace_size(cch.struct, 8, 0, f)
-            ws = torch.empty(nb, dtype=torch.uint8, device=device)
-            caches.append((cch, qn, kn, vn, out, ws, nb))
-        p = resa.params(0.1, 0, 0)
+        print(json.dumps({"mode": "rectify_sweep", **rectify_cell(T, f, device, peaks, peak_kind)}), flush=True)
 
-        def one(c):
-            cch, qn, kn, vn, out, ws, nb = c
-            resa.resa_rectify_attention(cch.struct, qn, kn, vn, f, p, out, None, ws, nb)
-            resa.resa_commit_kv(cch.struct, kn, vn, f, True)
 
-        def rect_only(c):
-            cch, qn, kn, vn, out, ws, nb = c
-            resa.resa_rectify_attention(cch.struct, qn, kn, vn, f, p, out, None, ws, nb)
-        for c in caches:
-            one(c)
-        torch.cuda.synchronize()
-        reps = max(2, math.ceil(8 / ncache))
-        g_all = capture(lambda: [one(c) for _ in range(reps) for c in caches], device)
-        g_rect = capture(lambda: [rect_only(c) for _ in range(reps) for c in caches], device)
-        g_all.replay()
-        g_rect.replay()
-        calls = reps * ncache
-        t_all = time_graph(g_all, 3) / calls
-        t_rect = time_graph(g_rect, 3) / calls
-        for c in caches:
-            code, _ = resa.resa_read_device_error(c[0].struct)
-            if code:
-                raise RuntimeError(f"device error {resa.DEVICE_ERRORS.get(code)}")
-        flops = rectify_flops(B, Hq, T, f)
-        byts = rectify_bytes(B, Hq, Hkv, T, f)
-        tf = flops / t_rect / 1e12
-        gbs = byts / t_rect / 1e9
-        line = {"mode": "rectify_sweep", "context": T, "f": f, "batch": B, "caches_rotated": ncache,
-                "rectify_us": round(t_rect * 1e6, 2), "rectify_plus_overwrite_us": round(t_all * 1e6, 2),
-                "TFLOP/s": round(tf, 1), "frac_bf16_burst": round(tf / float(peaks["bf16_tflops"]), 3),
-                "frac_bf16_sustained": round(tf / float(peaks["bf16_tflops_sustained"]), 3),
-                "GB/s": round(gbs, 1), "frac_hbm": round(gbs / float(peaks["hbm_gbs"]), 3),
-                "bound": "hbm" if 7 * f < float(peaks["bf16_tflops"]) / float(peaks["hbm_gbs"]) * 1e3 else "tensor",
-                "peak_kind": peak_kind}
-        print(json.dumps(line), flush=True)
-        del caches, g_all, g_rect
-        torch.cuda.empty_cache()
+TARGET_WORKLOAD = "qwen7b_b1_ctx256k_keep5"
+TARGET_LAYERS = 4
+TARGET_RECTIFY = ((262144, 32), (262144, 64))
+TARGET_DECODE_FRAC_HBM = 0.70
+TARGET_RECTIFY_FRAC_BF16 = 0.50
+
+
+def run_targets(device) -> dict:
+    """The two performance targets, measured after the headline (no oracle):
+    sparse decode at 256K context, batch 1, keep 0.05 (the decode call's
+    roofline fraction, the fused decode step per token, the rectify share of
+    the period), over TARGET_LAYERS rotated layer caches, per-call graphs
+    timed with CUDA events; and rectification at 256K with f = 32 and 64
+    against the burst bf16 peak (a call timed in isolation)."""
+    import torch
+    w = synth.WORKLOADS[TARGET_WORKLOAD]
+    peaks, peak_kind = load_peaks()
+    hbm = float(peaks["hbm_gbs"])
+    f, L, B = w.f, TARGET_LAYERS, w.batch
+    capacity = ((w.context + f * (2 + 2 * (1 + ATTR_REPS)) + BLOCK) // BLOCK + 1) * BLOCK
+    layers = [LayerCache(w, capacity, w.seed * 100 + 53 * i, device) for i in range(L)]
+    run_period(layers)                          # warm-up call outside any graph, appends f tokens
+    torch.cuda.synchronize()
+    T_attr = w.context + f
+    with ClockSampler(device.index or 0) as clocks:
+        mean_us, ncalls = time_call_kinds(layers, device)
+        cells = [rectify_cell(T, fr, device, peaks, peak_kind) for T, fr in TARGET_RECTIFY]
+    algo = call_bytes(w, T_attr)
+    dec_gbs = algo["decode"] / (mean_us["decode"] * 1e-6) / 1e9
+    period_us = sum(mean_us[k] * ncalls[k] for k in IN_STEP) / L     # one layer's period of f tokens
+    rect_us = (mean_us["rectify"] * ncalls["rectify"] + mean_us["overwrite"] * ncalls["overwrite"]) / L
+    del layers
+    torch.cuda.empty_cache()
+    rect = {}
+    for c in cells:
+        rect[f"f{c['f']}"] = {k: c[k] for k in ("rectify_us", "rectify_plus_overwrite_us", "TFLOP/s",
+                                                "frac_bf16_burst", "frac_bf16_sustained", "GB/s", "frac_hbm",
+                                                "bound")}
+    return {
+        "decode_256k": {
+            "workload": w.name, "batch": B, "context": T_attr, "keep": w.keep, "layers_rotated": L,
+            "decode_call_us": round(mean_us["decode"], 2), "decode_GB/s": round(dec_gbs, 1),
+            "decode_frac_hbm": round(dec_gbs / hbm, 3), "decode_algorithmic_bytes": int(algo["decode"]),
+            "target_frac_hbm": TARGET_DECODE_FRAC_HBM, "met": dec_gbs / hbm >= TARGET_DECODE_FRAC_HBM,
+            "select_call_us": round(mean_us["select"], 2),
+            "decode_step_us_per_token": round(mean_us["decode_step"], 2),
+            "us_per_token_with_rectify": round(period_us / f, 2),
+            "rectify_share_of_period": round(rect_us / period_us, 3),
+            "rectify_call_us": round(mean_us["rectify"], 2),
+            "decode_attention_latency_note": "per token of one layer: the fused decode step (append + select + "
+                                            "decode); with rectify and overwrite amortised over the f tokens in "
+                                            "us_per_token_with_rectify"},
+        "rectify_256k": {**rect, "target_frac_bf16_burst": TARGET_RECTIFY_FRAC_BF16,
+                         "met_f64": rect["f64"]["frac_bf16_burst"] >= TARGET_RECTIFY_FRAC_BF16,
+                         "peak_bf16_burst": float(peaks["bf16_tflops"])},
+        "peak_kind": peak_kind, "clocks": clocks.summary(),
+        "timing": "CUDA events around per-call-type CUDA graphs (decode: 4 rotated 256K caches; rectify: one "
+                  "537 MB cache per call, larger than L2), after the headline's timed region"}
 
 
 def run_breakdown(args):
@@ -913,6 +1043,8 @@ def main():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
     ap.add_argument("--layers", type=int, default=4, help="independent layer caches rotated per decode step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-targets", action="store_true",
+                    help="skip the 256K decode and rectify target measurements after the headline")
     ap.add_argument("--prefill", action="store_true", help="chunked dense prefill throughput (32K, 128K prompts)")
     ap.add_argument("--breakdown", action="store_true",
                     help="per-call latency breakdown versus dense decoding at 16K/64K/256K, batch 8")

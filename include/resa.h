@@ -147,6 +147,19 @@ resa_status_t resa_max_selected(const resa_cache_t* cache, const resa_params_t* 
 resa_status_t resa_decode_num_splits(const resa_cache_t* cache, int32_t n_cap, int32_t* splits_out);
 
 /*
+ * Number of key splits resa_rectify_attention uses for f new tokens on the
+ * current device (Section 2.2; the dense pass is split over the cached keys
+ * like Algorithm 2 splits the decode): the query rows of a KV head form
+ * ceil(8 f / 256) row groups of up to 256 rows (token-major, heads padded to
+ * 8), and splits = SMs / (batch * num_kv_heads * row groups), at least 1 and
+ * at most the 64-key tiles of the cache's capacity and 256. Split s of a
+ * sequence with T tokens takes the 64-key tiles [s * per, (s + 1) * per) of
+ * its prefix [0, T - f), per = ceil(ceil((T - f) / 64) / splits); the last
+ * split also takes the f new tokens.
+ */
+resa_status_t resa_rectify_num_splits(const resa_cache_t* cache, int32_t f, int32_t* splits_out);
+
+/*
  * Bytes of scratch workspace the compute calls need for this cache:
  * resa_select_blocks (block scores), resa_sparse_decode with `num_splits`
  * (0 = auto) at budget cap n_cap (split partials), and
@@ -304,6 +317,25 @@ resa_status_t resa_rectify_attention_active(const resa_cache_t* cache, const int
 resa_status_t resa_sparse_decode_static(const resa_cache_t* cache, const void* q, const int32_t* indices,
                                         const int32_t* counts, int32_t n_cap, const resa_params_t* params,
                                         void* out, float* lse, int32_t num_splits, void* stream);
+
+/*
+ * Failure-detection hook of the sparse decode kernel (resa_sparse_decode,
+ * resa_decode_step, resa_sparse_decode_static). Each warp of that kernel
+ * waits for the copies of its K/V blocks on shared-memory barriers, and
+ * gives up after `polls` polls of one barrier phase: it then records
+ * RESA_DEV_WAIT_TIMEOUT in device_status, skips its remaining blocks (the
+ * partial output covers the blocks attended before the wait ran out; a warp
+ * that attended none contributes nothing, so an output row whose every warp
+ * gave up is zero with lse -inf), and still waits, with the default limit,
+ * for every copy it had issued before its CTA exits, so no copy lands in
+ * released shared memory. The default, RESA_DEFAULT_DECODE_WAIT_POLLS, only
+ * runs out if a copy never completes; 0 makes every wait give up at once,
+ * which lets a test drive the timeout path without a fault or a hang. The
+ * setting is process-wide and read when a call is issued (a captured graph
+ * keeps the value of its capture). Always returns RESA_OK.
+ */
+#define RESA_DEFAULT_DECODE_WAIT_POLLS (1u << 22)
+resa_status_t resa_set_decode_wait_polls(uint32_t polls);
 
 /*
  * Synchronises `stream`, then copies device_status[0..1] to *code_out /

@@ -37,6 +37,12 @@ the CUDA path):
    their tokens (a min/max cannot be "un-applied").
 9. Rectified queries attend to the new (dense) K/V of the f tokens, causally:
    query i of the f sees positions [0, T - f + i].
+10. Non-finite values (the paper assumes finite ones): a NaN among a block's
+   valid keys makes that dimension of its Eq. 3 min and max NaN; a NaN
+   summary element or pooled-query element makes the Eq. 4 score NaN; in
+   Eq. 5 a NaN score ranks below every number, -inf included, and NaN scores
+   tie among themselves (lower block index first). Forced local blocks score
+   +inf whatever their summary holds.
 """
 from __future__ import annotations
 
@@ -104,14 +110,17 @@ def selection_budget(M: int, keep: float, n_min: int, n_local: int) -> int:
 def select_blocks(scores: np.ndarray, n: int, n_local: int) -> np.ndarray:
     """Top-n blocks after forcing the last n_local to +inf (Eq. 5 text).
 
-    Ranking: higher score first, ties to the lower block index. Returns the
-    selected block ids in ascending order.
+    Ranking: higher score first, a NaN score below every number (reading 10),
+    ties to the lower block index. Returns the selected block ids in
+    ascending order.
     """
     M = scores.shape[0]
     s = scores.astype(np.float64).copy()
     if n_local > 0:
         s[max(0, M - n_local):] = math.inf
-    order = np.lexsort((np.arange(M), -s))   # primary: -score, secondary: index
+    nan = np.isnan(s)
+    # primary: NaN last, then -score, then the block index
+    order = np.lexsort((np.arange(M), np.where(nan, 0.0, -s), nan))
     return np.sort(order[:n])
 
 

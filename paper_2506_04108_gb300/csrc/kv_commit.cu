@@ -10,6 +10,7 @@
 //               of its block and recomputes the block's summary from all of
 //               its valid keys (a min/max cannot be "un-applied").
 //  * bulk:      one warp per block recomputes Eq. 3 from the paged keys.
+// A NaN in a valid key makes that dimension of its block's min and max NaN.
 #include "resa_device.cuh"
 #include "resa_launch.h"
 
@@ -156,8 +157,8 @@ __global__ void __launch_bounds__(256) update_summaries_kernel(CacheView c, int 
   }
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
-    mn[j] = fminf(mn[j], __shfl_xor_sync(0xffffffffu, mn[j], 16));
-    mx[j] = fmaxf(mx[j], __shfl_xor_sync(0xffffffffu, mx[j], 16));
+    mn[j] = fmin_nan(mn[j], __shfl_xor_sync(0xffffffffu, mn[j], 16));
+    mx[j] = fmax_nan(mx[j], __shfl_xor_sync(0xffffffffu, mx[j], 16));
   }
   uint16_t* s = c.summ + summ_off(c, b, h, blk);
   if (half == 0)

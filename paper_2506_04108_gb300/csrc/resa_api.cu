@@ -23,6 +23,8 @@ constexpr size_t kAlign = 256;
 size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 std::atomic<int> g_sm_count[kMaxDevices];
+static_assert(RESA_DEFAULT_DECODE_WAIT_POLLS == (1u << 22), "the decode's default wait bound is the kernels' own");
+std::atomic<uint32_t> g_decode_wait_polls{RESA_DEFAULT_DECODE_WAIT_POLLS};
 
 resa_status_t sm_count(int* out) {
   int dev = 0;
@@ -238,6 +240,11 @@ const char* resa_status_string(resa_status_t s) {
   return "RESA_ERR_UNKNOWN";
 }
 
+resa_status_t resa_set_decode_wait_polls(uint32_t polls) {
+  g_decode_wait_polls.store(polls, std::memory_order_relaxed);
+  return RESA_OK;
+}
+
 resa_status_t resa_max_selected(const resa_cache_t* cache, const resa_params_t* params, int32_t* n_out) {
   resa_status_t s = check_cache(cache);
   if (s != RESA_OK) return s;
@@ -253,6 +260,17 @@ resa_status_t resa_decode_num_splits(const resa_cache_t* cache, int32_t n_cap, i
   if (n_cap <= 0 || splits_out == nullptr) return RESA_ERR_INVALID_ARG;
   int v = 0;
   if ((s = auto_decode_splits(cache, n_cap, &v)) != RESA_OK) return s;
+  *splits_out = v;
+  return RESA_OK;
+}
+
+resa_status_t resa_rectify_num_splits(const resa_cache_t* cache, int32_t f, int32_t* splits_out) {
+  resa_status_t s = check_cache(cache);
+  if (s != RESA_OK) return s;
+  if (f <= 0 || f > cache->max_blocks_per_seq * cache->block_size || splits_out == nullptr)
+    return RESA_ERR_INVALID_ARG;
+  int v = 0;
+  if ((s = auto_rectify_splits(cache, f, &v)) != RESA_OK) return s;
   *splits_out = v;
   return RESA_OK;
 }
@@ -353,7 +371,8 @@ resa_status_t resa_sparse_decode(const resa_cache_t* cache, const void* q, const
                                              align_up(rows * splits * kHeadDimHost * sizeof(float)));
   const cudaStream_t st = static_cast<cudaStream_t>(stream);
   cudaError_t e = launch_sparse_decode(view(cache), tk, tv, static_cast<const uint16_t*>(q), indices, counts, n_cap,
-                                       scale_of(cache, params), splits, o_part, lse_part, st);
+                                       scale_of(cache, params), splits, o_part, lse_part, st,
+                                       g_decode_wait_polls.load(std::memory_order_relaxed));
   if (e == cudaSuccess)
     e = launch_merge(o_part, lse_part, static_cast<int>(rows), splits, static_cast<uint16_t*>(out), lse, st);
   return e == cudaSuccess ? RESA_OK : RESA_ERR_CUDA;
@@ -396,7 +415,8 @@ resa_status_t resa_decode_step(const resa_cache_t* cache, const void* k_new, con
                                              align_up(rows * splits * kHeadDimHost * sizeof(float)));
   if (e == cudaSuccess)
     e = launch_sparse_decode(v, tk, tv, static_cast<const uint16_t*>(q), indices, counts, n_cap,
-                             scale_of(cache, params), splits, o_part, lse_part, st);
+                             scale_of(cache, params), splits, o_part, lse_part, st,
+                                       g_decode_wait_polls.load(std::memory_order_relaxed));
   if (e == cudaSuccess)
     e = launch_merge(o_part, lse_part, static_cast<int>(rows), splits, static_cast<uint16_t*>(out), lse, st, nullptr,
                      cache->num_q_heads, &v);
@@ -500,7 +520,8 @@ resa_status_t resa_sparse_decode_static(const resa_cache_t* cache, const void* q
                                              align_up(rows * splits * kHeadDimHost * sizeof(float)));
   const cudaStream_t st = static_cast<cudaStream_t>(stream);
   cudaError_t e = launch_sparse_decode(view(cache), tk, tv, static_cast<const uint16_t*>(q), indices, counts, n_cap,
-                                       scale_of(cache, params), splits, o_part, lse_part, st);
+                                       scale_of(cache, params), splits, o_part, lse_part, st,
+                                       g_decode_wait_polls.load(std::memory_order_relaxed));
   if (e == cudaSuccess)
     e = launch_merge(o_part, lse_part, static_cast<int>(rows), splits, static_cast<uint16_t*>(out), lse, st);
   return e == cudaSuccess ? RESA_OK : RESA_ERR_CUDA;

@@ -26,16 +26,30 @@ __device__ __forceinline__ void record_error(int32_t* status, int32_t code, int3
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
+// min / max that propagate NaN (PTX min.NaN / max.NaN; the result is the
+// canonical NaN if either input is NaN). Eq. 3 uses them: a NaN in any valid
+// key of a block makes that dimension of the block's summary NaN.
+__device__ __forceinline__ float fmin_nan(float a, float b) {
+  float d;
+  asm("min.NaN.f32 %0, %1, %2;" : "=f"(d) : "f"(a), "f"(b));
+  return d;
+}
+__device__ __forceinline__ float fmax_nan(float a, float b) {
+  float d;
+  asm("max.NaN.f32 %0, %1, %2;" : "=f"(d) : "f"(a), "f"(b));
+  return d;
+}
+
 // Folds 8 bf16 values (one 16-byte piece) into running fp32 min/max (Eq. 3).
 __device__ __forceinline__ void minmax8(const uint4& v, float* mn, float* mx) {
   const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
     const float lo = bf16_lo(w[i]), hi = bf16_hi(w[i]);
-    mn[2 * i] = fminf(mn[2 * i], lo);
-    mx[2 * i] = fmaxf(mx[2 * i], lo);
-    mn[2 * i + 1] = fminf(mn[2 * i + 1], hi);
-    mx[2 * i + 1] = fmaxf(mx[2 * i + 1], hi);
+    mn[2 * i] = fmin_nan(mn[2 * i], lo);
+    mx[2 * i] = fmax_nan(mx[2 * i], lo);
+    mn[2 * i + 1] = fmin_nan(mn[2 * i + 1], hi);
+    mx[2 * i + 1] = fmax_nan(mx[2 * i + 1], hi);
   }
 }
 
@@ -112,6 +126,13 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 // Bounded wait for phase `parity` of the barrier; false if it ran out.
 __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity) {
   for (uint32_t i = 0; i < kWaitPolls; ++i)
+    if (mbar_try_wait(bar, parity)) return true;
+  return false;
+}
+
+// The same with a caller-chosen number of polls (0: give up at once).
+__device__ __forceinline__ bool mbar_wait_polls(uint32_t bar, uint32_t parity, uint32_t polls) {
+  for (uint32_t i = 0; i < polls; ++i)
     if (mbar_try_wait(bar, parity)) return true;
   return false;
 }

@@ -81,9 +81,13 @@ cudaError_t launch_select(const CacheView& c, const uint16_t* q, double keep, in
 
 // sparse_decode.cu
 int decode_ctas_per_sm();  // resident decode CTAs per SM (occupancy), >= 1
+// `wait_polls`: polls of one copy's barrier before a warp gives up
+// (RESA_DEV_WAIT_TIMEOUT); copies already issued are then still awaited with
+// the default limit before the CTA exits.
 cudaError_t launch_sparse_decode(const CacheView& c, const CUtensorMap& tm_k, const CUtensorMap& tm_v,
                                  const uint16_t* q, const int32_t* indices, const int32_t* counts, int n_cap,
-                                 float sm_scale, int splits, float* o_part, float* lse_part, cudaStream_t st);
+                                 float sm_scale, int splits, float* o_part, float* lse_part, cudaStream_t st,
+                                 uint32_t wait_polls);
 // `advance` (a fused decode step's view, pending > 0): the merge also counts
 // the appended token in seq_lens; rows_per_seq must then be Hq.
 cudaError_t launch_merge(const float* o_part, const float* lse_part, int rows, int splits, uint16_t* out,

@@ -44,10 +44,11 @@ constexpr int kTopnCtaWarps = kTopnCtaThreads / 32;
 constexpr int kTopnCtaMaxBlocks = 6144;  // the one-CTA form serves caches up to this many blocks per sequence
 static_assert(kTopnCtaMaxBlocks * sizeof(uint32_t) <= 48 * 1024, "one-CTA top-n keys fit the default shared memory");
 
-// Exact max of two packed bf16 pairs.
+// Exact max of two packed bf16 pairs; NaN propagates (a NaN summary element
+// makes the block's score NaN).
 __device__ __forceinline__ uint32_t bf16x2_max(uint32_t a, uint32_t b) {
   uint32_t d;
-  asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  asm("max.NaN.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
   return d;
 }
 
@@ -340,8 +341,11 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c,
 }
 
 // Order-preserving map of an fp32 score to uint32 (larger score, larger key).
+// A NaN score maps to 0, below every number (-inf maps to 0x007FFFFF): NaN
+// blocks rank last, among themselves by block index like every tie.
 __device__ __forceinline__ uint32_t score_key(float s) {
   const uint32_t u = __float_as_uint(s);
+  if ((u & 0x7FFFFFFFu) > 0x7F800000u) return 0u;
   return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
@@ -460,11 +464,11 @@ __device__ __forceinline__ void push_v2(uint32_t dst, uint32_t x, uint32_t y, ui
 // The select stops early when the boundary bucket is taken whole. Then each
 // CTA counts its keys above the boundary and at it; every warp reads the
 // counts of the lower-ranked CTAs and of the lower warps and writes its
-// selected ids in ascending order (ties at the boundary to the lower id). A
-// CTA leaves once it holds all its parts: no peer writes to it afterwards.
-// A wait that runs out records RESA_DEV_WAIT_TIMEOUT; the thread then writes
-// no ids and waits at a cluster barrier (which completes once every other
-// thread has arrived or exited) before it leaves.
+// selected ids in ascending order (ties at the boundary to the lower id).
+// A wait that runs out records RESA_DEV_WAIT_TIMEOUT; the CTA then pushes
+// nothing more and writes no ids. Every thread of every CTA arrives at one
+// closing cluster barrier after its CTA's last push and waits on it just
+// before it leaves, whether its waits succeeded or not.
 // 40 registers (3 CTAs per SM): a CTA launched early then fits beside the
 // persistent score CTA (88 registers x 512 threads), so its prologue runs
 // before the scores are complete.
@@ -681,9 +685,15 @@ __global__ void __launch_bounds__(kTopnThreads, 3) topn_kernel(CacheView c, cons
   const int s_in = warp_incl_scan(s_l);
   int eq_seen = eq_before + __shfl_sync(0xffffffffu, e_ex, warp);
   int pos = sel_before + __shfl_sync(0xffffffffu, s_in - s_l, warp);
+  // Closing cluster barrier, split: every thread arrives here, after its
+  // CTA's last push, and waits just before it leaves, on the success and the
+  // failure path alike, so no CTA leaves while a peer may still push into its
+  // shared memory (a CTA that timed out stops pushing, but its peers may not
+  // have noticed yet).
+  asm volatile("barrier.cluster.arrive.release;" ::: "memory");
   if (failed) {  // (warp-uniform) values received may be incomplete: write no ids
     if (lane == 0) record_error(c.status, RESA_DEV_WAIT_TIMEOUT, b * c.Hkv + h);
-    asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+    asm volatile("barrier.cluster.wait.acquire;" ::: "memory");
     return;
   }
   for (int i0 = w0; i0 < w1; i0 += 32) {
@@ -700,6 +710,7 @@ __global__ void __launch_bounds__(kTopnThreads, 3) topn_kernel(CacheView c, cons
   }
   for (int i = n + static_cast<int>(rank) * kTopnThreads + tid; i < n_cap; i += kTopnCluster * kTopnThreads) out[i] = -1;
   if (rank == 0 && tid == 0) counts[b * c.Hkv + h] = n;
+  asm volatile("barrier.cluster.wait.acquire;" ::: "memory");
 }
 
 // One-CTA radix select, grid (KV head, sequence), for caches of up to

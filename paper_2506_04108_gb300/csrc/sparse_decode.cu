@@ -42,6 +42,7 @@ struct DecodeArgs {
   float scale_log2;
   float* o_part;    // [B][Hq][splits][128]
   float* lse_part;  // [B][Hq][splits], log2 domain
+  uint32_t wait_polls;  // polls of a copy's barrier before the warp gives up (the drain keeps kWaitPolls)
 };
 
 __device__ __forceinline__ float safe_base(float m) { return m == kNegInf ? 0.f : m; }
@@ -152,7 +153,7 @@ __global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid
     const uint32_t par = (it / kStages) & 1;
     const uint32_t bar = bar0 + 8 * st;
     int ok = 1;
-    if (lane == 0) ok = mbar_wait_bounded(bar, par) ? 1 : 0;
+    if (lane == 0) ok = mbar_wait_polls(bar, par, a.wait_polls) ? 1 : 0;
     ok = __shfl_sync(0xffffffffu, ok, 0);
     if (!ok) {
       if (lane == 0) record_error(c.status, RESA_DEV_WAIT_TIMEOUT, b * c.Hkv + h);
@@ -230,7 +231,7 @@ __global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid
       ++issued;
     }
   }
-  if (it < cnt && lane == 0) {  // timed out: let copies already in flight land before leaving
+  if (it < cnt && lane == 0) {  // timed out: let copies already in flight land (default limit) before leaving
     for (int k = it; k < issued; ++k) mbar_wait_bounded(bar0 + 8 * (k % kStages), (k / kStages) & 1);
   }
 
@@ -412,10 +413,12 @@ int decode_ctas_per_sm() {
 
 cudaError_t launch_sparse_decode(const CacheView& c, const CUtensorMap& tm_k, const CUtensorMap& tm_v,
                                  const uint16_t* q, const int32_t* indices, const int32_t* counts, int n_cap,
-                                 float sm_scale, int splits, float* o_part, float* lse_part, cudaStream_t st) {
+                                 float sm_scale, int splits, float* o_part, float* lse_part, cudaStream_t st,
+                                 uint32_t wait_polls) {
   cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(sparse_decode_kernel), kDecodeSmem, 0);
   if (e != cudaSuccess) return e;
-  DecodeArgs a{q, indices, counts, n_cap, splits, sm_scale * 1.44269504088896340736f, o_part, lse_part};
+  DecodeArgs a{q,        indices,  counts, n_cap, splits, sm_scale * 1.44269504088896340736f,
+               o_part,   lse_part, wait_polls};
   return launch_pdl(sparse_decode_kernel, dim3(splits, c.Hkv, c.B), dim3(kWarps * 32), kDecodeSmem, st, tm_k,
                     tm_v, c, a);
 }

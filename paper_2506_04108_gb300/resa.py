@@ -27,7 +27,9 @@ DEVICE_ERRORS = {0: "RESA_DEV_OK", 1: "RESA_DEV_SEQ_LEN_RANGE", 2: "RESA_DEV_PAG
 EXPORTED = ["resa_abi_version", "resa_status_string", "resa_max_selected", "resa_decode_num_splits",
             "resa_workspace_size", "resa_update_summaries", "resa_commit_kv", "resa_select_blocks",
             "resa_sparse_decode", "resa_rectify_attention", "resa_read_device_error", "resa_sparse_decode_static",
-            "resa_commit_kv_active", "resa_rectify_attention_active", "resa_decode_step"]
+            "resa_commit_kv_active", "resa_rectify_attention_active", "resa_decode_step",
+            "resa_rectify_num_splits", "resa_set_decode_wait_polls"]
+DEFAULT_DECODE_WAIT_POLLS = 1 << 22
 
 
 class ResaError(RuntimeError):
@@ -66,6 +68,8 @@ def load() -> ctypes.CDLL:
         "resa_status_string": ([c_int32], ctypes.c_char_p),
         "resa_max_selected": ([cp, pc, POINTER(c_int32)], c_int32),
         "resa_decode_num_splits": ([cp, c_int32, POINTER(c_int32)], c_int32),
+        "resa_rectify_num_splits": ([cp, c_int32, POINTER(c_int32)], c_int32),
+        "resa_set_decode_wait_polls": ([ctypes.c_uint32], c_int32),
         "resa_workspace_size": ([cp, c_int32, c_int32, c_int32, POINTER(c_size_t)], c_int32),
         "resa_update_summaries": ([cp, c_int32, c_int32, pp], c_int32),
         "resa_commit_kv": ([cp, pp, pp, c_int32, c_int32, pp], c_int32),
@@ -129,6 +133,18 @@ def resa_decode_num_splits(cache: ResaCacheT, n_cap: int) -> int:
     s = c_int32(0)
     _check(load().resa_decode_num_splits(ctypes.byref(cache), n_cap, ctypes.byref(s)), "resa_decode_num_splits")
     return s.value
+
+
+def resa_rectify_num_splits(cache: ResaCacheT, f: int) -> int:
+    s = c_int32(0)
+    _check(load().resa_rectify_num_splits(ctypes.byref(cache), f, ctypes.byref(s)), "resa_rectify_num_splits")
+    return s.value
+
+
+def resa_set_decode_wait_polls(polls: int = DEFAULT_DECODE_WAIT_POLLS):
+    """Polls of one copy barrier after which the sparse decode kernel gives up
+    (RESA_DEV_WAIT_TIMEOUT); process-wide. 0 makes every wait give up at once."""
+    _check(load().resa_set_decode_wait_polls(int(polls)), "resa_set_decode_wait_polls")
 
 
 def resa_workspace_size(cache: ResaCacheT, n_cap: int, num_splits: int = 0, max_f: int = 0) -> int:

@@ -128,17 +128,27 @@ def round_bf16(x: np.ndarray) -> np.ndarray:
 
 
 def check_outputs(gpu, ref, what=""):
-    """GPU outputs are bf16 (the C ABI's output type), so they are compared
-    with the oracle's fp64 result rounded to bf16: the tolerance then bounds
-    the kernel's arithmetic, not the output format's quantisation (about
-    ulp/4 = 1e-3 mean for |O| ~ 1). The max-abs bound also holds against the
-    unrounded fp64 result."""
+    """GPU outputs are bf16 (the C ABI's output type); the oracle's are fp64.
+
+    * max-abs <= 2e-2 against the unrounded fp64 result and against it
+      rounded to bf16;
+    * mean-abs <= 1e-3 against the fp64 result rounded to bf16 (the kernel's
+      arithmetic error alone);
+    * mean-abs against the unrounded fp64 result <= 1e-3 plus the mean error
+      that rounding the exact result to bf16 itself leaves (ulp/4 on average:
+      ~2e-3 for outputs of magnitude 1, ~1e-4 for the small outputs of long
+      contexts): a bf16 output cannot do better than its own rounding.
+    """
     gpu = np.asarray(gpu, dtype=np.float64)
     ref = np.asarray(ref, dtype=np.float64)
     assert np.isfinite(gpu).all(), f"{what}: non-finite output"
+    rounded = round_bf16(ref)
     raw = np.abs(gpu - ref)
-    err = np.abs(gpu - round_bf16(ref))
+    err = np.abs(gpu - rounded)
+    floor = np.abs(rounded - ref).mean()
     assert raw.max() <= OUT_MAX_ABS, f"{what}: max-abs vs fp64 {raw.max():.3e} > {OUT_MAX_ABS}"
     assert err.max() <= OUT_MAX_ABS, f"{what}: max-abs {err.max():.3e} > {OUT_MAX_ABS}"
     assert err.mean() <= OUT_MEAN_ABS, f"{what}: mean-abs {err.mean():.3e} > {OUT_MEAN_ABS}"
+    assert raw.mean() <= OUT_MEAN_ABS + floor, \
+        f"{what}: mean-abs vs fp64 {raw.mean():.3e} > {OUT_MEAN_ABS} + bf16 rounding floor {floor:.3e}"
     return float(err.max()), float(err.mean())

@@ -105,6 +105,16 @@ def test_bad_call_arguments_rejected_on_host(lib):
     assert step(k=0) == 1 and step(v=0) == 1 and step(q=0) == 1 and step(out=0) == 1
     assert step(v=0x71008) == 1 and step(n_cap=0) == 1 and step(splits=-1) == 1 and step(splits=2000) == 1
     assert step(wsb=16) == 3 and step(ws=0) == 3
+    # split query of the rectification: f outside [1, capacity] or no output pointer
+    n = ctypes.c_int32(0)
+    assert lib.resa_rectify_num_splits(cp, 0, ctypes.byref(n)) == 1
+    assert lib.resa_rectify_num_splits(cp, 32 * 16 + 1, ctypes.byref(n)) == 1
+    assert lib.resa_rectify_num_splits(cp, 8, None) == 1
+
+
+def test_decode_wait_limit_setter_needs_no_device(lib):
+    assert lib.resa_set_decode_wait_polls(0) == 0
+    assert lib.resa_set_decode_wait_polls(resa.DEFAULT_DECODE_WAIT_POLLS) == 0
 
 
 @pytest.mark.parametrize("max_blocks,keep,n_min,n_local", [(256, 0.1, 16, 4), (2048, 0.1, 128, 1),

@@ -146,6 +146,63 @@ def test_topn_exhaustive_subset_maximises_score_sum():
         assert O.select_blocks(scores, n, 0).tolist() == sorted(best)
 
 
+# ------------------------------------------- non-finite values (reading 10) ---
+def test_summary_nan_key_poisons_only_its_dimension():
+    """A NaN key makes its block's min and max NaN in that dimension only; the
+    online update agrees with the recompute (brute force over the other dims)."""
+    g = synth.rng(71)
+    b, d, T = 16, 6, 40
+    K = rand_bf16(g, (T, d))
+    K[20, 2] = np.nan                     # block 1, dimension 2
+    kmin, kmax = O.block_summaries(K, b)
+    for i in range(3):
+        for j in range(d):
+            vals = K[i * b:min(T, (i + 1) * b), j]
+            if i == 1 and j == 2:
+                assert np.isnan(kmin[i, j]) and np.isnan(kmax[i, j])
+            else:
+                assert kmin[i, j] == min(vals.tolist()) and kmax[i, j] == max(vals.tolist())
+    st = O.SequenceState(1, 48, d, b)
+    for t in range(T):
+        st.append(K[None, t], K[None, t])
+    assert np.array_equal(st.kmin[0, :3], kmin, equal_nan=True)
+    assert np.array_equal(st.kmax[0, :3], kmax, equal_nan=True)
+
+
+def test_score_nan_from_summary_or_query():
+    g = synth.rng(72)
+    kmin, kmax = O.block_summaries(rand_bf16(g, (64, 8)), 16)
+    q = g.standard_normal(8)
+    kmin[2, 5] = np.nan
+    s = O.quest_scores(q, kmin, kmax)
+    assert np.isnan(s[2]) and np.isfinite(np.delete(s, 2)).all()
+    q[0] = np.nan
+    assert np.isnan(O.quest_scores(q, kmin, kmax)).all()
+
+
+def test_topn_nan_ranks_last_brute_force():
+    """A block is kept iff fewer than n blocks beat it, where a number beats
+    NaN, a larger number beats a smaller one, and within equal scores (NaN
+    with NaN included) the lower index wins; forced blocks score +inf."""
+    g = synth.rng(73)
+    for trial in range(300):
+        M = int(g.integers(1, 14))
+        scores = np.round(g.standard_normal(M) * 2) / 2
+        scores[g.random(M) < 0.3] = np.nan
+        scores[g.random(M) < 0.1] = -np.inf
+        n_local = int(g.integers(0, 4))
+        n = int(g.integers(max(1, min(n_local, M)), M + 1))
+        eff = [math.inf if i >= M - n_local else scores[i] for i in range(M)]
+
+        def beats(j, i):
+            a, c = eff[j], eff[i]
+            if math.isnan(a) or math.isnan(c):
+                return (not math.isnan(a)) or (math.isnan(c) and j < i)
+            return a > c or (a == c and j < i)
+        want = [i for i in range(M) if sum(1 for j in range(M) if j != i and beats(j, i)) < n]
+        assert O.select_blocks(scores, n, n_local).tolist() == want
+
+
 # --------------------------------------------------------- Eq. 1 / Eq. 2 ---
 def test_two_key_softmax_worked():
     ex = GOLDEN["two_key_softmax"]
