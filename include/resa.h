@@ -306,8 +306,11 @@ resa_status_t resa_rectify_attention_active(const resa_cache_t* cache, const int
  *     (batch * num_q_heads * splits * (head_dim + 1) * 4 bytes, each part
  *     rounded up to 256 bytes) return RESA_ERR_WORKSPACE and launch nothing.
  *   - The first call on a device looks up the buffer's device address (with
- *     that device current) and caches it; make that first call before any
- *     stream capture on that device.
+ *     that device current) and caches it for the rest of the process; make
+ *     that first call before any stream capture on that device. The cached
+ *     address belongs to the device's primary context: after cudaDeviceReset
+ *     (or anything else that destroys that context) it is stale, and this
+ *     entry point must not be called again in that process.
  *   - All calls share the one buffer, and it keeps the last call's contents
  *     (nothing in it needs to start at zero: every call overwrites every
  *     partial it reads). Calls that overlap on the GPU (e.g. on two streams
