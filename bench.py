@@ -834,7 +834,10 @@ def run_rectify_sweep(args):
     device = torch.device("cuda", 0)
     torch.cuda.set_device(0)
     peaks, peak_kind = load_peaks()
-    for T, f in synth.RECTIFY_SWEEP:
+    cells = synth.RECTIFY_SWEEP
+    if args.rectify_cells:
+        cells = [tuple(int(x) for x in cell.split(":")) for cell in args.rectify_cells.split(",")]
+    for T, f in cells:
         print(json.dumps({"mode": "rectify_sweep", **rectify_cell(T, f, device, peaks, peak_kind)}), flush=True)
 
 
@@ -1050,6 +1053,8 @@ def main():
                     help="per-call latency breakdown versus dense decoding at 16K/64K/256K, batch 8")
     ap.add_argument("--rectify-sweep", action="store_true",
                     help="time rectification over the 16K/64K/256K x f 16/32/64 grid instead")
+    ap.add_argument("--rectify-cells", default=None,
+                    help="with --rectify-sweep: only these cells, 'context:f' comma-separated (e.g. 65536:64)")
     ap.add_argument("--oracle-worker", default=None, help=argparse.SUPPRESS)
     ap.add_argument("--repeats", type=int, default=1, help=argparse.SUPPRESS)
     ap.add_argument("--min-seconds", type=float, default=0.0, help=argparse.SUPPRESS)
