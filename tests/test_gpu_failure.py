@@ -148,3 +148,52 @@ def test_nan_key_appended_poisons_its_block_summary():
         assert np.array_equal(summ[0, h, :M, 0], mn, equal_nan=True)
         assert np.array_equal(summ[0, h, :M, 1], mx, equal_nan=True)
     assert np.isnan(summ[0, 0, 2, 0, 7]) and np.isnan(summ[0, 0, 2, 1, 7])
+
+
+def test_nan_key_appended_by_the_fused_step():
+    """The fused decode step folds the appended key into its block's summary
+    inside the score kernel (Eq. 3 online update): a NaN key poisons that
+    dimension there too, the block (the forced local one) is still selected,
+    and the output of its group is NaN while the other group stays finite and
+    matches the oracle."""
+    g, Hkv, T = 4, 2, 300
+    gr = synth.rng(7400)
+    K = synth.normal_bf16(gr, (Hkv, T, 128))
+    V = synth.normal_bf16(gr, (Hkv, T, 128))
+    cache = H.make_cache([K], [V], g * Hkv, (T + 1 + 15) // 16 + 1)
+    p = resa.params(0.1, 4, 1)
+    n_cap = resa.resa_max_selected(cache.struct, p)
+    kn = synth.normal_bf16(gr, (1, Hkv, 128))
+    vn = synth.normal_bf16(gr, (1, Hkv, 128))
+    kn[0, 1, 5] = BF16_NAN                       # KV head 1's appended key
+    q = synth.normal_bf16(gr, (1, g * Hkv, 128))
+    idx = torch.empty((1, Hkv, n_cap), dtype=torch.int32, device="cuda")
+    cnt = torch.empty((1, Hkv), dtype=torch.int32, device="cuda")
+    out = torch.empty((1, g * Hkv, 128), dtype=torch.bfloat16, device="cuda")
+    ws, nb = H.workspace(cache, n_cap)
+    resa.resa_decode_step(cache.struct, H.dev_bf16(kn), H.dev_bf16(vn), H.dev_bf16(q), p, idx, cnt, n_cap, out, None,
+                          0, ws, nb)
+    assert resa.resa_read_device_error(cache.struct) == (0, 0)
+    assert int(cache.seq_lens[0]) == T + 1
+    Kall = np.concatenate([K, kn[0][:, None]], axis=1)
+    Vall = np.concatenate([V, vn[0][:, None]], axis=1)
+    summ = H.host_f64(cache.summaries)[0]
+    M = (T + 1 + 15) // 16
+    for h in range(Hkv):
+        mn, mx = O.block_summaries(O.widen_bf16(Kall[h]), 16)
+        assert np.array_equal(summ[h, :M, 0], mn, equal_nan=True)
+        assert np.array_equal(summ[h, :M, 1], mx, equal_nan=True)
+    idx, cnt, out = idx.cpu().numpy(), cnt.cpu().numpy(), H.host_f64(out)
+    for h in range(Hkv):
+        mn, mx = O.block_summaries(O.widen_bf16(Kall[h]), 16)
+        qg = O.widen_bf16(q[0, h * g:(h + 1) * g])
+        scores = O.quest_scores(O.pooled_query(qg), mn, mx)
+        n = O.selection_budget(M, 0.1, 4, 1)
+        sel = idx[0, h, :cnt[0, h]]
+        H.check_selection(sel, scores, n, 1)
+        assert M - 1 in sel.tolist()
+        o, _ = O.gbsa_attention(qg, O.widen_bf16(Kall[h]), O.widen_bf16(Vall[h]), T + 1, sel, 16, SCALE)
+        if h == 1:
+            assert np.isnan(o).all() and np.isnan(out[0, h * g:(h + 1) * g]).all()
+        else:
+            H.check_outputs(out[0, h * g:(h + 1) * g], o, "fused step, finite group")
