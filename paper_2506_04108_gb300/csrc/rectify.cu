@@ -13,13 +13,15 @@
 // (normalised O, log2-sum-exp) are combined by merge_kernel.
 //
 // CTA = 12 warps:
-//   warp 0      TMA producer: 64-key K and V tiles of the prefix, one
-//               SWIZZLE_128B box per 16-key page per 64-column half, issued
-//               by 16 lanes, into a 5-stage ring (kv_full / kv_empty
-//               mbarriers); page ids are read 32 blocks at a time. The
-//               tiles of the f new tokens come from k_new / v_new by 4-D TMA
-//               boxes (64 tokens x 64 dims of one head), only up to the last
-//               token of the CTA's rows (later keys are causally masked).
+//   warps 0, 2, 3  TMA producers: 64-key K and V tiles of the prefix, one
+//               SWIZZLE_128B box per 16-key page per 64-column half (16 per
+//               tile, spread over the three warps: copies issued by the lanes
+//               of one warp go out one after another), into a 5-stage ring
+//               (kv_full / kv_empty mbarriers); page ids are read 32 blocks at
+//               a time. The tiles of the f new tokens come from k_new / v_new
+//               by 4-D TMA boxes (64 tokens x 64 dims of one head), only up to
+//               the last token of the CTA's rows (later keys are causally
+//               masked).
 //   warp 1      allocates 512 TMEM columns; lane 0 issues the MMAs:
 //               S[t] = Q K^T (M 128, N 64, K 128; both operands K-major from
 //               shared memory) into a double-buffered TMEM S, and
@@ -180,10 +182,15 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
   fence_proxy_async_smem();
   __syncthreads();
 
-  if (warp == 0) {
-    // ------------------------------------------------------- producer ---
-    // Page rows of the prefix blocks are read 32 at a time (8 tiles, one
-    // block per lane) and the 16 boxes of a tile are issued by 16 lanes.
+  if (warp == 0 || warp == 2 || warp == 3) {
+    // ------------------------------------------------------ producers ---
+    // Three warps issue the boxes of each tile (TMA copies issued by the
+    // lanes of one warp go out one after another; separate warps issue in
+    // parallel): box j of a prefix tile (page j / 4, part j % 4: K or V, one
+    // 64-column half) is issued by producer j % 3; warp 0 also posts the
+    // stage's byte count. Page rows of the prefix blocks are read 32 at a
+    // time (eight tiles).
+    const int pw = warp == 0 ? 0 : warp - 1;  // producer 0, 1, 2
     int win = -1, my_row = -1;
     for (int t = 0; t < n_tiles; ++t) {
       const int st = t % kStages;
@@ -201,32 +208,35 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
             const int page = c.page_table[static_cast<size_t>(b) * c.max_blocks + blk];
             if (page >= 0 && page < c.num_pages)
               my_row = (page * c.Hkv + h) * kBlock;
-            else if (win * (kTileKeys / kBlock) + lane < n_pref * (kTileKeys / kBlock))
+            else if (pw == 0 && win * (kTileKeys / kBlock) + lane < n_pref * (kTileKeys / kBlock))
               record_error(c.status, RESA_DEV_PAGE_RANGE, b);  // a block this CTA uses: left out
           }
         }
         const int slot = (t - win) * (kTileKeys / kBlock);
-        int pages = 0;
+        if (pw == 0) {
+          int pages = 0;
 #pragma unroll
-        for (int pg = 0; pg < kTileKeys / kBlock; ++pg) pages += __shfl_sync(0xffffffffu, my_row, slot + pg) >= 0 ? 1 : 0;
-        const int row = __shfl_sync(0xffffffffu, my_row, slot + ((lane >> 2) & 3));
-        if (lane == 0) mbar_arrive_expect_tx(bar(kBarKvFull + st), pages * 4 * 2048);
-        __syncwarp();
-        if (lane < 16 && row >= 0) {  // lane 4 pg + part: part 0/1 = K halves, 2/3 = V halves
-          const int part = lane & 3;
-          tma_load_2d(kdst + part * kKVHalf + (lane >> 2) * 2048, part < 2 ? &tm_k : &tm_v, bar(kBarKvFull + st),
+          for (int pg = 0; pg < kTileKeys / kBlock; ++pg) pages += __shfl_sync(0xffffffffu, my_row, slot + pg) >= 0 ? 1 : 0;
+          if (lane == 0) mbar_arrive_expect_tx(bar(kBarKvFull + st), pages * 4 * 2048);
+        }
+        // this producer's boxes j = pw + 3 l (lane l), j < 16
+        const int j = pw + 3 * lane;
+        const int row = __shfl_sync(0xffffffffu, my_row, slot + ((j >> 2) & 3));
+        if (j < 16 && row >= 0) {
+          const int part = j & 3;
+          tma_load_2d(kdst + part * kKVHalf + (j >> 2) * 2048, part < 2 ? &tm_k : &tm_v, bar(kBarKvFull + st),
                       (part & 1) * 64, row);
         }
       } else {
         // tail tile: tokens tb .. tb + 63 of the f new ones, by TMA from
-        // k_new / v_new viewed as [B][f][Hkv][128] (tokens >= f read as zero)
+        // k_new / v_new viewed as [B][f][Hkv][128] (tokens >= f read as zero);
+        // producer pw issues boxes pw and (pw == 0) 3
         const int tb = (t - n_pref) * kTileKeys;
         if (lane == 0) {
-          mbar_arrive_expect_tx(bar(kBarKvFull + st), 4 * kKVHalf);
-          tma_load_4d(kdst, &tm_kn, bar(kBarKvFull + st), 0, h, tb, b);
-          tma_load_4d(kdst + kKVHalf, &tm_kn, bar(kBarKvFull + st), 64, h, tb, b);
-          tma_load_4d(kdst + 2 * kKVHalf, &tm_vn, bar(kBarKvFull + st), 0, h, tb, b);
-          tma_load_4d(kdst + 3 * kKVHalf, &tm_vn, bar(kBarKvFull + st), 64, h, tb, b);
+          if (pw == 0) mbar_arrive_expect_tx(bar(kBarKvFull + st), 4 * kKVHalf);
+          for (int part = pw; part < 4; part += 3)
+            tma_load_4d(kdst + part * kKVHalf, part < 2 ? &tm_kn : &tm_vn, bar(kBarKvFull + st), (part & 1) * 64, h,
+                        tb, b);
         }
       }
     }
