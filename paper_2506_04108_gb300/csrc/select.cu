@@ -4,10 +4,9 @@
 //               (small caches: 4 KB) pieces of the block summaries with its
 //               own bulk copies through its own shared-memory ring and
 //               scores them with the pooled query of the piece's GQA group
-//               (mean of the g heads, fp32); a
-//               half-warp takes one block, a lane one 16-byte piece (8 dims)
-//               of k_min and k_max, and the 128-dim sum is a fixed-order
-//               butterfly over the 16 lanes.
+//               (mean of the g heads, fp32); eight lanes take one block, a
+//               lane 16 dims of k_min and k_max, and the 128-dim sum is a
+//               fixed-order butterfly over the 8 lanes.
 // top-n        one CTA (caches of up to kTopnCtaMaxBlocks blocks per
 //               sequence) or one 8-CTA cluster (larger caches) per (sequence,
 //               KV head). The n of Eq. 5 is evaluated on the device from the
@@ -42,32 +41,35 @@ constexpr int kTopnSmemMax = 200 * 1024;                           // staged key
 constexpr int kTopnCtaThreads = 512;                                // one-CTA form
 constexpr int kTopnCtaWarps = kTopnCtaThreads / 32;
 constexpr int kTopnCtaMaxBlocks = 6144;  // the one-CTA form serves caches up to this many blocks per sequence
-static_assert(kTopnCtaMaxBlocks * sizeof(uint32_t) <= 48 * 1024, "one-CTA top-n keys fit the default shared memory");
+constexpr int kTopnCtaKeys = kTopnCtaMaxBlocks / kTopnCtaThreads;   // keys held per thread
+static_assert(kTopnCtaKeys * kTopnCtaThreads == kTopnCtaMaxBlocks && kTopnCtaKeys <= 32, "one-CTA key layout");
 
-// Exact max of two packed bf16 pairs; NaN propagates (a NaN summary element
-// makes the block's score NaN).
-__device__ __forceinline__ uint32_t bf16x2_max(uint32_t a, uint32_t b) {
-  uint32_t d;
-  asm("max.NaN.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
-  return d;
-}
-
-// Eq. 4 partial sum over 8 dims. Per dimension max(q k_max, q k_min) equals
-// |q| max(s k_max, s k_min) with s = sign(q) (scaling by |q| >= 0 and the fp32
-// rounding are monotone, so the max is taken exactly); the sign is applied to
-// the bf16 bits (`sg`), the max of two bf16 values is exact, and one fp32 FMA
-// per dimension accumulates |q| times it.
-__device__ __forceinline__ float quest_term8(const float* qa, const uint32_t* sg, const uint4& mn, const uint4& mx) {
+// Eq. 4 partial sum over 8 dims, accumulated into s. Since k_min <= k_max in
+// every dimension, max(q k_max, q k_min) is q k_max where q >= 0 and q k_min
+// where q < 0 (sign bit set): one byte permute per bf16 pair picks the factor
+// (`sel`, from the signs of the pooled query), and one fp32 FMA per dimension
+// accumulates q times it. The product is the one the max would return, bit
+// for bit (infinities and a zero q included); a NaN key makes both k_min and
+// k_max NaN in its dimension, so the picked factor is NaN either way.
+__device__ __forceinline__ float quest_term8(const float* qf, const uint32_t* sel, const uint4& mn, const uint4& mx,
+                                             float s) {
   const uint32_t a[4] = {mn.x, mn.y, mn.z, mn.w};
   const uint32_t c[4] = {mx.x, mx.y, mx.z, mx.w};
-  float s = 0.f;
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    const uint32_t m = bf16x2_max(a[i] ^ sg[i], c[i] ^ sg[i]);
-    s = fmaf(qa[2 * i], bf16_lo(m), s);
-    s = fmaf(qa[2 * i + 1], bf16_hi(m), s);
+    const uint32_t m = __byte_perm(a[i], c[i], sel[i]);
+    s = fmaf(qf[2 * i], bf16_lo(m), s);
+    s = fmaf(qf[2 * i + 1], bf16_hi(m), s);
   }
   return s;
+}
+
+// __byte_perm selector for one bf16 pair (low element first): bytes of k_min
+// (0-3) where the query element's sign bit is set, of k_max (4-7) elsewhere.
+__device__ __forceinline__ uint32_t quest_selector(float q_lo, float q_hi) {
+  const uint32_t lo = signbit(q_lo) ? 0x0010u : 0x0054u;
+  const uint32_t hi = signbit(q_hi) ? 0x3200u : 0x7600u;
+  return lo | hi;
 }
 
 // Persistent score kernel: one CTA per SM. The (sequence, KV head) units'
@@ -77,13 +79,16 @@ __device__ __forceinline__ float quest_term8(const float* qa, const uint32_t* sg
 // streams its pieces with 1-D bulk copies issued by its own lane 0 through
 // its own kScoreStages-stage shared-memory ring: copies issued by one thread
 // complete one after another, so sixteen independent issuers keep enough
-// bytes in flight per SM. Two shapes, the same 192 KB of rings: 12-block
+// bytes in flight per SM. Every stage is filled before the dependency wait,
+// and a warp refills a stage as soon as it has scored it (lane 0 locates the
+// refill's piece while it waits for the stage's copy). Two shapes, the same 192 KB of rings: 12-block
 // (6 KB) pieces in 2 stages when the cache has at least one such piece per
 // warp of the grid (measured: they beat 8 blocks in 3 stages, and 16 blocks
 // with 12 warps, at 32K x 8 and 256K x 1), else 8-block (4 KB) pieces in 3
-// stages, which give more warps a piece. A half-warp scores one block, a
-// lane one 16-byte piece (8 dims) of k_min and k_max, and the 128-dim sum
-// ends in a fixed-order 16-lane butterfly.
+// stages, which give more warps a piece. Eight lanes score one block, a lane
+// 16 dims of k_min and k_max (two 16-byte chunks, dims 8c..8c+7 and
+// 64+8c..64+8c+7 for lane c of the eight), and the 128-dim sum ends in a
+// fixed-order 8-lane butterfly.
 constexpr int kScoreWarps = 16;
 constexpr int kMaxBatch = 1024;  // sequences per call supported by the score kernel
 constexpr int score_piece_bytes(int piece_blocks) { return piece_blocks * 2 * kHeadDim * 2; }
@@ -96,10 +101,14 @@ constexpr int score_smem_bytes(int piece_blocks, int stages) {
 }
 constexpr int score_table_bytes(int B) { return (3 * B + 1) * static_cast<int>(sizeof(int)); }
 
+// At most 88 registers: a score CTA (512 x 88) then fits beside one merge
+// CTA (256 x 64), so that one launched early issues its first copies while
+// the preceding step's merge runs, and a top-n cluster CTA launched early
+// (512 x 40) fits beside a score CTA.
 template <int kPieceBlocks, int kScoreStages>
-__global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c, const uint16_t* __restrict__ q,
+__global__ void __maxnreg__(88) score_kernel(CacheView c, const uint16_t* __restrict__ q,
                                                                     float* __restrict__ scores) {
-  static_assert(kPieceBlocks % 2 == 0, "two half-warps score a piece's blocks in pairs");
+  static_assert(kPieceBlocks % 4 == 0, "four lane groups score a piece's blocks four at a time");
   constexpr int kPieceBytes = score_piece_bytes(kPieceBlocks);
   constexpr int kScoreRing = score_ring_bytes(kPieceBlocks, kScoreStages);
   constexpr int kScoreSmem = score_smem_bytes(kPieceBlocks, kScoreStages);
@@ -181,15 +190,22 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c,
     nmine = ncta > warp ? (ncta - warp + kScoreWarps - 1) / kScoreWarps : 0;
   };
   my_range();
-  auto issue = [&](int k) {  // lane 0: this warp's k-th piece into stage (kbase + k) % kScoreStages
+  struct Src {
+    const uint16_t* p;
+    uint32_t bytes;
+  };
+  auto piece_src = [&](int k) {  // this warp's k-th piece: its summaries and size
     int b, h, blk0, nblk;
     locate(c0 + warp + k * kScoreWarps, b, h, blk0, nblk);
-    const uint32_t bar = bar0 + 8 * ((kbase + k) % kScoreStages);
-    const uint32_t bytes = static_cast<uint32_t>(nblk) * 2 * kHeadDim * 2;
-    mbar_arrive_expect_tx(bar, bytes);
-    bulk_load(ring_s + ((kbase + k) % kScoreStages) * kPieceBytes,
-              c.summ + ((static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks + blk0) * 2 * kHeadDim, bytes, bar);
+    return Src{c.summ + ((static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks + blk0) * 2 * kHeadDim,
+               static_cast<uint32_t>(nblk) * 2 * kHeadDim * 2};
   };
+  auto issue_src = [&](int k, const Src& src) {  // lane 0: piece k into stage (kbase + k) % kScoreStages
+    const uint32_t bar = bar0 + 8 * ((kbase + k) % kScoreStages);
+    mbar_arrive_expect_tx(bar, src.bytes);
+    bulk_load(ring_s + ((kbase + k) % kScoreStages) * kPieceBytes, src.p, src.bytes, bar);
+  };
+  auto issue = [&](int k) { issue_src(k, piece_src(k)); };
   __syncwarp();  // lane 0's barrier initialisation precedes every lane's use
   if (lane == 0)
     for (int k = 0; k < min(kScoreStages, nmine); ++k) issue(k);
@@ -218,49 +234,57 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c,
       for (int k = 0; k < min(kScoreStages, nmine); ++k) issue(k);
   }
 
-  const int ch = lane & 15, half = lane >> 4;
+  const int ch = lane & 15, half = lane >> 4;  // the appended token: a lane folds 8 dims
+  const int c8 = lane & 7, grp = lane >> 3;     // scoring: lane c8 of group grp
   int cur_unit = -1, k_fail = -1;
-  float qa[8];
-  uint32_t sg[4];
+  float qf[16];
+  uint32_t sel[8];
   uint4 ka = make_uint4(0, 0, 0, 0), va = ka;  // the appended token's key / value, this lane's 8 dims
   for (int k = 0; k < nmine; ++k) {
     const int st = (kbase + k) % kScoreStages, par = ((kbase + k) / kScoreStages) & 1;
     int b, h, blk0, nblk;
     locate(c0 + warp + k * kScoreWarps, b, h, blk0, nblk);
     const int unit = b * c.Hkv + h;
-    if (unit != cur_unit) {  // pooled query (mean of the group's heads), this lane's 8 dims
+    if (unit != cur_unit) {  // pooled query (mean of the group's heads), this lane's 16 dims
       cur_unit = unit;
       if (c.pending) {
         const size_t kv = (static_cast<size_t>(b) * c.Hkv + h) * kHeadDim + ch * 8;
         ka = *reinterpret_cast<const uint4*>(c.k_append + kv);
         va = *reinterpret_cast<const uint4*>(c.v_append + kv);
       }
-      float qp[8];
+      // this lane's dims 8 c8 .. 8 c8 + 7 (part 0) and 64 + 8 c8 .. 64 + 8 c8 + 7
+      // (part 1): lane group grp adds heads grp and grp + 4, and two butterfly
+      // levels over the four groups complete the sum of the g heads
+      const uint16_t* qg = q + (static_cast<size_t>(b) * c.Hq + h * c.g) * kHeadDim + c8 * 8;
+      uint4 qv[4];  // head grp parts 0, 1; head grp + 4 parts 0, 1 (g <= 8)
 #pragma unroll
-      for (int j = 0; j < 8; ++j) qp[j] = 0.f;
-      const uint16_t* qg = q + (static_cast<size_t>(b) * c.Hq + h * c.g) * kHeadDim + ch * 8;
-      uint4 qv[kMaxGroup];  // all g rows in flight at once (g <= 8)
+      for (int i = 0; i < 4; ++i) {
+        const int head = grp + 4 * (i >> 1);
+        qv[i] = head < c.g ? *reinterpret_cast<const uint4*>(qg + head * kHeadDim + 64 * (i & 1)) : make_uint4(0, 0, 0, 0);
+      }
 #pragma unroll
-      for (int i = 0; i < kMaxGroup; ++i)
-        qv[i] = i < c.g ? *reinterpret_cast<const uint4*>(qg + i * kHeadDim) : make_uint4(0, 0, 0, 0);
-#pragma unroll
-      for (int i = 0; i < kMaxGroup; ++i) {
-        const uint32_t w[4] = {qv[i].x, qv[i].y, qv[i].z, qv[i].w};
+      for (int part = 0; part < 2; ++part) {
+        const uint32_t w0[4] = {qv[part].x, qv[part].y, qv[part].z, qv[part].w};
+        const uint32_t w1[4] = {qv[2 + part].x, qv[2 + part].y, qv[2 + part].z, qv[2 + part].w};
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-          qp[2 * j] += bf16_lo(w[j]);
-          qp[2 * j + 1] += bf16_hi(w[j]);
+          qf[8 * part + 2 * j] = bf16_lo(w0[j]) + bf16_lo(w1[j]);
+          qf[8 * part + 2 * j + 1] = bf16_hi(w0[j]) + bf16_hi(w1[j]);
         }
       }
       const float inv_g = 1.0f / static_cast<float>(c.g);
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const float lo = qp[2 * j] * inv_g, hi = qp[2 * j + 1] * inv_g;
-        qa[2 * j] = fabsf(lo);
-        qa[2 * j + 1] = fabsf(hi);
-        sg[j] = ((__float_as_uint(lo) >> 16) & 0x8000u) | (__float_as_uint(hi) & 0x80000000u);
+      for (int j = 0; j < 16; ++j) {
+        qf[j] += __shfl_xor_sync(0xffffffffu, qf[j], 8);
+        qf[j] += __shfl_xor_sync(0xffffffffu, qf[j], 16);
+        qf[j] *= inv_g;
       }
+#pragma unroll
+      for (int j = 0; j < 8; ++j) sel[j] = quest_selector(qf[2 * j], qf[2 * j + 1]);
     }
+    // lane 0 locates the piece that refills this stage before waiting for it
+    const bool issue_next = lane == 0 && k + kScoreStages < nmine;
+    const Src next = issue_next ? piece_src(k + kScoreStages) : Src{nullptr, 0u};
     int ok = 1;
     if (lane == 0) ok = mbar_wait_bounded(bar0 + 8 * st, par) ? 1 : 0;
     ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -312,24 +336,25 @@ __global__ void __launch_bounds__(kScoreWarps * 32, 1) score_kernel(CacheView c,
     }
     float* out = scores + static_cast<size_t>(unit) * c.max_blocks + blk0;
 #pragma unroll
-    for (int v = 0; v < kPieceBlocks / 2; ++v) {
-      const int blk = 2 * v + half;
+    for (int v = 0; v < kPieceBlocks / 4; ++v) {
+      const int blk = 4 * v + grp;
       float sc = 0.f;
       if (blk < nblk) {
-        const uint4 mn = *reinterpret_cast<const uint4*>(piece + blk * 512 + ch * 16);
-        const uint4 mx = *reinterpret_cast<const uint4*>(piece + blk * 512 + 256 + ch * 16);
-        sc = quest_term8(qa, sg, mn, mx);
+        const uint8_t* pb = piece + blk * 512 + c8 * 16;
+        const uint4 mn0 = *reinterpret_cast<const uint4*>(pb), mn1 = *reinterpret_cast<const uint4*>(pb + 128);
+        const uint4 mx0 = *reinterpret_cast<const uint4*>(pb + 256), mx1 = *reinterpret_cast<const uint4*>(pb + 384);
+        sc = quest_term8(qf, sel, mn0, mx0, sc);
+        sc = quest_term8(qf + 8, sel + 4, mn1, mx1, sc);
       }
-      sc += __shfl_xor_sync(0xffffffffu, sc, 8);
       sc += __shfl_xor_sync(0xffffffffu, sc, 4);
       sc += __shfl_xor_sync(0xffffffffu, sc, 2);
       sc += __shfl_xor_sync(0xffffffffu, sc, 1);
-      if (ch == 0 && blk < nblk) out[blk] = sc;
+      if (c8 == 0 && blk < nblk) out[blk] = sc;
     }
     __syncwarp();  // every lane has read the stage before it is refilled
-    if (lane == 0 && k + kScoreStages < nmine) {
+    if (issue_next) {
       fence_proxy_async_smem();
-      issue(k + kScoreStages);
+      issue_src(k + kScoreStages, next);
     }
   }
   // A warp that gave up may have copies in flight (pieces k_fail .. k_fail + kScoreStages - 1):
@@ -715,17 +740,19 @@ __global__ void __launch_bounds__(kTopnThreads, 3) topn_kernel(CacheView c, cons
 
 // One-CTA radix select, grid (KV head, sequence), for caches of up to
 // kTopnCtaMaxBlocks blocks per sequence: the same selection as topn_kernel
-// with every barrier a CTA barrier. The histograms rotate through three
-// buffers, so one barrier per pass suffices (the buffer zeroed during a pass
-// was last read two passes before); warp 0 finds each digit and one more
-// barrier hands it to the other warps. The ordered compaction gives each warp
-// a contiguous id range, and every warp derives its output offset from the
-// per-warp counts after a single barrier.
-__global__ void __launch_bounds__(kTopnCtaThreads, 1) topn_cta_kernel(CacheView c, const float* __restrict__ scores,
+// with every barrier a CTA barrier. Warp w owns the contiguous id range
+// [w * per_warp, (w + 1) * per_warp) and its lane l the ids w * per_warp +
+// 32 j + l, whose keys it keeps in registers from staging to compaction: a
+// pass reads no shared memory but the histogram, and its shared-memory
+// atomics are independent of one another. The histograms rotate through
+// three buffers, so one barrier per pass suffices (the buffer zeroed during a
+// pass was last read two passes before); warp 0 finds each digit and one
+// more barrier hands it to the other warps. Every warp derives its output
+// offset from the per-warp counts after a single barrier.
+__global__ void __launch_bounds__(kTopnCtaThreads, 2) topn_cta_kernel(CacheView c, const float* __restrict__ scores,
                                                                       double keep, int n_min, int n_local,
                                                                       int32_t* __restrict__ indices,
                                                                       int32_t* __restrict__ counts, int n_cap) {
-  extern __shared__ uint32_t keys[];
   __shared__ __align__(16) int hist[3][256];
   __shared__ uint32_t w_lo[kTopnCtaWarps], w_hi[kTopnCtaWarps];
   __shared__ int w_gt[kTopnCtaWarps], w_eq[kTopnCtaWarps];
@@ -747,51 +774,44 @@ __global__ void __launch_bounds__(kTopnCtaThreads, 1) topn_cta_kernel(CacheView 
   }
   const UnitBudget u = unit_budget(T, keep, n_min, n_local, n_cap, c.status, b * c.Hkv + h, tid == 0);
   const int M = u.M, n = u.n, F = u.F, nf = u.nf, r = u.r;
-  const float* sc = scores + (static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks;
+  const int per_warp = ((M + 31) / 32 + kTopnCtaWarps - 1) / kTopnCtaWarps * 32;  // <= 32 kTopnCtaKeys
+  const int w0 = warp * per_warp;
+  // bit j: id w0 + 32 j + lane is a candidate (< F) / a forced block taken ([F, F + nf))
+  uint32_t cand = 0, forced = 0;
+#pragma unroll
+  for (int j = 0; j < kTopnCtaKeys; ++j) {
+    const int i = w0 + 32 * j + lane;
+    if (32 * j < per_warp) {
+      if (i < F) cand |= 1u << j;
+      else if (i - F < nf) forced |= 1u << j;
+    }
+  }
+  const float* sc = scores + (static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks + w0 + lane;
   pdl_wait();  // the scores
   pdl_launch_dependents();  // after the wait: see the score kernel
+  uint32_t key[kTopnCtaKeys];
+#pragma unroll
+  for (int j = 0; j < kTopnCtaKeys; ++j) key[j] = (cand >> j) & 1u ? score_key(sc[32 * j]) : 0u;
   uint32_t kmin = 0xFFFFFFFFu, kmax = 0u;
-  // one round of loads for up to 4096 blocks (a unit of 32K tokens holds 2049)
-  constexpr int kLoads = 8;
-  for (int i0 = 0; i0 < M; i0 += kLoads * kTopnCtaThreads) {
-    float v[kLoads];
 #pragma unroll
-    for (int k = 0; k < kLoads; ++k) {
-      const int i = i0 + k * kTopnCtaThreads + tid;
-      v[k] = i < M ? sc[i] : 0.f;
+  for (int j = 0; j < kTopnCtaKeys; ++j)
+    if ((cand >> j) & 1u) {
+      kmin = min(kmin, key[j]);
+      kmax = max(kmax, key[j]);
     }
-#pragma unroll
-    for (int k = 0; k < kLoads; ++k) {
-      const int i = i0 + k * kTopnCtaThreads + tid;
-      if (i < M) {
-        const uint32_t key = score_key(v[k]);
-        keys[i] = key;
-        if (i < F) {
-          kmin = min(kmin, key);
-          kmax = max(kmax, key);
-        }
-      }
-    }
-  }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    kmin = min(kmin, __shfl_xor_sync(0xffffffffu, kmin, o));
-    kmax = max(kmax, __shfl_xor_sync(0xffffffffu, kmax, o));
-  }
+  kmin = __reduce_min_sync(0xffffffffu, kmin);
+  kmax = __reduce_max_sync(0xffffffffu, kmax);
   if (lane == 0) {
     w_lo[warp] = kmin;
     w_hi[warp] = kmax;
   }
-  __syncthreads();  // the keys and the per-warp extremes are visible
-  kmin = lane < kTopnCtaWarps ? w_lo[lane] : 0xFFFFFFFFu;
-  kmax = lane < kTopnCtaWarps ? w_hi[lane] : 0u;
+  __syncthreads();  // the per-warp extremes are visible
+  kmin = __reduce_min_sync(0xffffffffu, lane < kTopnCtaWarps ? w_lo[lane] : 0xFFFFFFFFu);
+  kmax = __reduce_max_sync(0xffffffffu, lane < kTopnCtaWarps ? w_hi[lane] : 0u);
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    kmin = min(kmin, __shfl_xor_sync(0xffffffffu, kmin, o));
-    kmax = max(kmax, __shfl_xor_sync(0xffffffffu, kmax, o));
-  }
+  for (int j = 0; j < kTopnCtaKeys; ++j) key[j] -= kmin;  // v = key - min key (candidates only are read)
 
-  // ---- radix select of the r-th largest v = key - kmin among blocks [0, F) ----
+  // ---- radix select of the r-th largest v among blocks [0, F) ----
   uint32_t prefix = 0, pmask = 0;
   int rem = r;
   if (r > 0 && r < F) {
@@ -800,11 +820,10 @@ __global__ void __launch_bounds__(kTopnCtaThreads, 1) topn_cta_kernel(CacheView 
     for (int pass = 0;; ++pass) {
       const uint32_t dmask = (1u << width) - 1u;
       int* hb = hist[pass % 3];
-      for (int i = tid; i < 256; i += kTopnCtaThreads) hist[(pass + 1) % 3][i] = 0;
-      for (int i = tid; i < F; i += kTopnCtaThreads) {
-        const uint32_t v = keys[i] - kmin;
-        if ((v & pmask) == prefix) atomicAdd(&hb[(v >> shift) & dmask], 1);
-      }
+      if (tid < 256) hist[(pass + 1) % 3][tid] = 0;
+#pragma unroll
+      for (int j = 0; j < kTopnCtaKeys; ++j)
+        if (((cand >> j) & 1u) && (key[j] & pmask) == prefix) atomicAdd(&hb[(key[j] >> shift) & dmask], 1);
       __syncthreads();  // this pass's histogram is complete
       if (warp == 0) {
         const DigitPick pk = pick_digit(hb, rem);
@@ -823,31 +842,18 @@ __global__ void __launch_bounds__(kTopnCtaThreads, 1) topn_cta_kernel(CacheView 
       shift -= width;
     }
   }
-  // Selected: forced blocks [F, F + nf), and among [0, F) the ids with
+  // Selected: the forced blocks, and among the candidates the ids with
   // (v & pmask) > prefix, or == prefix among the first `take_eq` such ids.
   const int take_eq = rem;
-  auto classify = [&](int i, bool in, bool& is_gt, bool& is_eq) {
-    is_gt = false;
-    is_eq = false;
-    if (in) {
-      if (i >= F) {
-        is_gt = i - F < nf;
-      } else {
-        const uint32_t v = (keys[i] - kmin) & pmask;
-        is_gt = v > prefix;
-        is_eq = v == prefix;
-      }
+  uint32_t gtm = forced, eqm = 0;
+#pragma unroll
+  for (int j = 0; j < kTopnCtaKeys; ++j)
+    if ((cand >> j) & 1u) {
+      const uint32_t v = key[j] & pmask;
+      if (v > prefix) gtm |= 1u << j;
+      else if (v == prefix) eqm |= 1u << j;
     }
-  };
-  const int per_warp = ((M + 31) / 32 + kTopnCtaWarps - 1) / kTopnCtaWarps * 32;
-  const int w0 = warp * per_warp, w1 = min(M, w0 + per_warp);
-  int gt = 0, eq = 0;
-  for (int i0 = w0; i0 < w1; i0 += 32) {
-    bool is_gt, is_eq;
-    classify(i0 + lane, i0 + lane < w1, is_gt, is_eq);
-    gt += __popc(__ballot_sync(0xffffffffu, is_gt));
-    eq += __popc(__ballot_sync(0xffffffffu, is_eq));
-  }
+  const int gt = __reduce_add_sync(0xffffffffu, __popc(gtm)), eq = __reduce_add_sync(0xffffffffu, __popc(eqm));
   if (lane == 0) {
     w_gt[warp] = gt;
     w_eq[warp] = eq;
@@ -855,32 +861,22 @@ __global__ void __launch_bounds__(kTopnCtaThreads, 1) topn_cta_kernel(CacheView 
   __syncthreads();  // every warp's counts are visible
   // this warp's offsets: equal keys and selected ids of the lower warps
   const int e_l = lane < kTopnCtaWarps ? w_eq[lane] : 0, g_l = lane < kTopnCtaWarps ? w_gt[lane] : 0;
-  int ie = e_l;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const int y = __shfl_up_sync(0xffffffffu, ie, o);
-    if (lane >= o) ie += y;
-  }
+  const int ie = warp_incl_scan(e_l);
   const int s_l = g_l + max(0, min(e_l, take_eq - (ie - e_l)));
-  int is = s_l;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const int y = __shfl_up_sync(0xffffffffu, is, o);
-    if (lane >= o) is += y;
-  }
+  const int is = warp_incl_scan(s_l);
   int eq_seen = __shfl_sync(0xffffffffu, ie - e_l, warp);
   int pos = __shfl_sync(0xffffffffu, is - s_l, warp);
-  for (int i0 = w0; i0 < w1; i0 += 32) {
-    const int i = i0 + lane;
-    bool is_gt, is_eq;
-    classify(i, i < w1, is_gt, is_eq);
-    const unsigned eqm = __ballot_sync(0xffffffffu, is_eq);
-    const int my_eq_rank = eq_seen + __popc(eqm & ((1u << lane) - 1u));
-    const bool sel = is_gt || (is_eq && my_eq_rank < take_eq);
-    const unsigned selm = __ballot_sync(0xffffffffu, sel);
-    if (sel) out[pos + __popc(selm & ((1u << lane) - 1u))] = i;
-    eq_seen += __popc(eqm);
-    pos += __popc(selm);
+  const unsigned below = (1u << lane) - 1u;
+#pragma unroll
+  for (int j = 0; j < kTopnCtaKeys; ++j) {
+    if (32 * j >= per_warp) break;
+    const bool is_eq = (eqm >> j) & 1u;
+    const unsigned eqb = __ballot_sync(0xffffffffu, is_eq);
+    const bool sel = ((gtm >> j) & 1u) || (is_eq && eq_seen + __popc(eqb & below) < take_eq);
+    const unsigned selb = __ballot_sync(0xffffffffu, sel);
+    if (sel) out[pos + __popc(selb & below)] = w0 + 32 * j + lane;
+    eq_seen += __popc(eqb);
+    pos += __popc(selb);
   }
   for (int i = n + tid; i < n_cap; i += kTopnCtaThreads) out[i] = -1;
   if (tid == 0) counts[b * c.Hkv + h] = n;
@@ -889,7 +885,7 @@ __global__ void __launch_bounds__(kTopnCtaThreads, 1) topn_cta_kernel(CacheView 
 }  // namespace
 
 size_t select_smem_bytes(int max_blocks) {
-  if (max_blocks <= kTopnCtaMaxBlocks) return static_cast<size_t>(max_blocks) * sizeof(uint32_t);
+  if (max_blocks <= kTopnCtaMaxBlocks) return 0;  // keys in registers
   return static_cast<size_t>((max_blocks + kTopnCluster - 1) / kTopnCluster) * sizeof(uint32_t);
 }
 
