@@ -187,6 +187,26 @@ def test_select_large_unit():
     check_select_case(cache, Ks, Vs, q, p, maxb, idx, cnt)
 
 
+@pytest.mark.parametrize("M", [6144, 5121])
+def test_select_one_cta_at_its_size_bound(M):
+    """The one-CTA top-n at the largest cache it serves: 6144 blocks fill all
+    twelve key slots of every thread; 5121 blocks leave the last warp with no
+    ids and the one before it with a partial range. Some blocks repeat, so
+    ties at the boundary are resolved by index."""
+    T = M * 16 - 5
+    gk = synth.rng(76)
+    K = synth.normal_bf16(gk, (1, T, 128))
+    K[:, 16 * 100:16 * 400] = np.tile(K[:, 16 * 99:16 * 100], (1, 300, 1))   # 300 identical blocks
+    V = synth.normal_bf16(gk, (1, T, 128))
+    cache = H.make_cache([K], [V], 7, M)
+    q = synth.normal_bf16(synth.rng(77), (1, 7, 128))
+    p = resa.params(0.1, 16, 2)
+    n_cap = resa.resa_max_selected(cache.struct, p)
+    idx, cnt = run_select(cache, q, p, n_cap)
+    assert resa.resa_read_device_error(cache.struct) == (0, 0)
+    check_select_case(cache, [K], [V], q, p, M, idx, cnt)
+
+
 @pytest.mark.parametrize("maxb", [44, 6200])  # one-CTA and cluster top-n
 def test_select_ties_go_to_lower_index(maxb):
     """Identical blocks give identical scores; the lower ids must win."""
