@@ -25,6 +25,7 @@ that type in step order, timed with CUDA events (total / calls).
 from __future__ import annotations
 
 import argparse
+import datetime
 import hashlib
 import json
 import math
@@ -127,9 +128,12 @@ def profiled_traffic(call: str, workload: str, src_hash: str):
 
 
 class ClockSampler:
-    """nvidia-smi clock / throttle sampling during the timed region."""
+    """nvidia-smi clock / throttle sampling every 20 ms. Between begin() and
+    end() (host times bracketing a synchronised timed region) only the
+    samples taken inside that window are summarised; without a window, or if
+    none fell inside it, all of them are, and the summary says which."""
 
-    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    QUERY = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
@@ -137,6 +141,14 @@ class ClockSampler:
         self.gpu_index = gpu_index
         self.proc = None
         self.path = None
+        self.window = None
+
+    def begin(self):
+        self.window = [datetime.datetime.now(), None]
+
+    def end(self):
+        if self.window is not None:
+            self.window[1] = datetime.datetime.now()
 
     def __enter__(self):
         try:
@@ -144,7 +156,7 @@ class ClockSampler:
             os.close(fd)
             self.fh = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu_index), f"--query-gpu={self.QUERY}",
-                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                          "--format=csv,noheader,nounits", "-lms", "20"],
                                          stdout=self.fh, stderr=subprocess.DEVNULL)
             time.sleep(0.3)
         except (OSError, FileNotFoundError):
@@ -163,26 +175,29 @@ class ClockSampler:
     def summary(self):
         if self.proc is None or self.path is None:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
-        sm, smax, reasons = [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        rows = []
         with open(self.path) as fh:
             for line in fh:
                 parts = [p.strip() for p in line.split(",")]
-                if len(parts) < 9:
+                if len(parts) < 10:
                     continue
                 try:
-                    sm.append(float(parts[1]))
-                    smax.append(float(parts[2]))
+                    t = datetime.datetime.strptime(parts[0], "%Y/%m/%d %H:%M:%S.%f")
+                    rows.append((t, float(parts[2]), float(parts[3]),
+                                 {nm for nm, v in zip(names, parts[6:10]) if v.lower() == "active"}))
                 except ValueError:
                     continue
-                for nm, v in zip(names, parts[5:9]):
-                    if v.lower() == "active":
-                        reasons.add(nm)
         os.unlink(self.path)
-        if not sm:
+        scope = "all samples"
+        if self.window is not None and self.window[1] is not None:
+            inside = [r for r in rows if self.window[0] <= r[0] <= self.window[1]]
+            if inside:
+                rows, scope = inside, "timed region"
+        if not rows:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
-                "samples": len(sm)}
+        return {"sm_mhz": statistics.median(r[1] for r in rows), "sm_max_mhz": max(r[2] for r in rows),
+                "reasons": sorted(set().union(*(r[3] for r in rows))), "samples": len(rows), "window": scope}
 
 
 # --------------------------------------------------------------- distributed
@@ -574,12 +589,14 @@ def run_ours(args, w: synth.Workload):
     with ClockSampler(local) as clocks:
         barrier()
         torch.cuda.synchronize()
+        clocks.begin()
         s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         s0.record()
         for _ in range(args.steps):
             graph.replay()
         s1.record()
         torch.cuda.synchronize()
+        clocks.end()
         barrier()
     T += f * args.steps
     secs = s0.elapsed_time(s1) / 1e3

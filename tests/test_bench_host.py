@@ -81,3 +81,29 @@ def test_oracle_worker_times_whole_periods_until_min_seconds():
     assert len(times) >= 2 and all(t > 0 for t in times)
     assert sum(times) >= 0.5 or len(times) == bench.ORACLE_MAX_REPEATS
     assert sum(times[:-1]) < 0.5 or len(times) == 2  # stops at the first period past the bound
+
+
+def test_clock_summary_keeps_the_timed_window(tmp_path):
+    """The clock summary uses only the samples inside begin()/end() when any
+    fell there (an idle sample before the region and a throttled one after it
+    are left out), and all of them otherwise."""
+    import datetime as dt
+    t0 = dt.datetime(2026, 1, 2, 3, 4, 5)
+    rows = [(t0, 1200, ""), (t0 + dt.timedelta(seconds=1), 2070, ""), (t0 + dt.timedelta(seconds=1.02), 2070, ""),
+            (t0 + dt.timedelta(seconds=3), 1500, "Active")]
+
+    def sampler(window):
+        path = tmp_path / f"clk{window is not None}.csv"
+        with open(path, "w") as fh:
+            for t, mhz, slow in rows:
+                fh.write(f"{t:%Y/%m/%d %H:%M:%S.%f}, 0, {mhz}, 2070, 900.0, 0x0, "
+                         f"{slow or 'Not Active'}, Not Active, Not Active, Not Active\n")
+        c = bench.ClockSampler(0)
+        c.proc, c.path, c.window = object(), str(path), window
+        return c.summary()
+
+    inside = sampler([t0 + dt.timedelta(seconds=0.5), t0 + dt.timedelta(seconds=2)])
+    assert inside == {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": [], "samples": 2, "window": "timed region"}
+    everything = sampler(None)
+    assert everything["samples"] == 4 and everything["window"] == "all samples"
+    assert everything["reasons"] == ["hw_slowdown"] and everything["sm_mhz"] == 1785.0
