@@ -116,6 +116,9 @@ def run_select(cache, q_bits, p, n_cap):
     (8, 1, [300, 5000], 0.05, 3, 2),
     (7, 4, [100, 80], 0.5, 16, 1),         # M <= n: every block selected
     (2, 2, [160], 0.0, 0, 12),             # n_local >= n
+    (3, 2, [300, 900], 0.2, 4, 1),         # group sizes 3, 5, 6: the pooled query's
+    (5, 2, [700], 0.2, 4, 1),              # head sum is split over four lane groups
+    (6, 1, [1200], 0.1, 0, 2),             # (heads j and j + 4)
 ])
 def test_select_matches_oracle(g, Hkv, lens, keep, n_min, n_local, wide):
     Ks, Vs = seq_inputs(5 + len(lens), len(lens), Hkv, lens)
