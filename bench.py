@@ -667,6 +667,11 @@ def run_ours(args, w: synth.Workload):
                "sample": f"1 of {B} sequences x 1 of {L} layers: {f} decode steps + 1 rectification at context "
                          f"{w.context}, timed {len(times)} times (fp64 numpy, 1 BLAS thread)",
                "seconds": round(secs_cpu, 3)}
+        # informational: the same oracle with its BLAS pool on every host core
+        ncores = os.cpu_count() or 1
+        times_all = run_oracle_subprocess(sample, threads=ncores, min_seconds=CPU_BASELINE_ALL_SECONDS)
+        cpu["all_cores"] = {"value": round(f * len(times_all) / sum(times_all), 2), "unit": UNIT, "cores": ncores,
+                            "seconds": round(sum(times_all), 3), "note": "informational; the baseline is 1 thread"}
 
     launches = args.steps * L * (f * LayerCache.KERNELS_PER_DECODE_STEP + LayerCache.KERNELS_PER_RECTIFY)
     line = {"metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -686,6 +691,7 @@ def run_ours(args, w: synth.Workload):
 
 ATTR_REPS = 3
 CPU_BASELINE_SECONDS = 10.0  # oracle work timed for cpu_baseline (whole periods, at least one)
+CPU_BASELINE_ALL_SECONDS = 5.0    # the informational all-cores timing of the same sample
 ORACLE_MAX_REPEATS = 400
 TOPN_CTA_MAX_BLOCKS = 6144  # caches of up to this many blocks per sequence use the one-CTA top-n
 
