@@ -566,6 +566,8 @@ def run_ours(args, w: synth.Workload):
     _b.build()
     resa.load()
 
+    if args.layers is None:
+        args.layers = max(4, w.layers)
     L, f, B = args.layers, w.f, w.batch
     # periods that append f tokens: warm-up call, graph warm-up/timed/e2e replays, attribution commits
     periods_total = 1 + args.warmup + args.steps + (2 + args.steps) + 2 * (1 + ATTR_REPS) + 1
@@ -1088,7 +1090,9 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
-    ap.add_argument("--layers", type=int, default=4, help="independent layer caches rotated per decode step")
+    ap.add_argument("--layers", type=int, default=None,
+                    help="independent layer caches rotated per decode step (default: the workload's layer count, "
+                         "at least 4)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-targets", action="store_true",
                     help="skip the 256K decode and rectify target measurements after the headline")
@@ -1113,6 +1117,8 @@ def main():
     if args.warmup < 3 and args.impl == "ours":
         ap.error("--warmup must be >= 3")
     w = synth.WORKLOADS[args.workload]
+    if args.layers is None:
+        args.layers = max(4, w.layers)
     if args.rectify_sweep:
         run_rectify_sweep(args)
         return
