@@ -749,6 +749,7 @@ __global__ void __launch_bounds__(kTopnThreads, 3) topn_kernel(CacheView c, cons
 // pass was last read two passes before); warp 0 finds each digit and one
 // more barrier hands it to the other warps. Every warp derives its output
 // offset from the per-warp counts after a single barrier.
+template <int kKeys>
 __global__ void __launch_bounds__(kTopnCtaThreads, 2) topn_cta_kernel(CacheView c, const float* __restrict__ scores,
                                                                       double keep, int n_min, int n_local,
                                                                       int32_t* __restrict__ indices,
@@ -774,12 +775,12 @@ __global__ void __launch_bounds__(kTopnCtaThreads, 2) topn_cta_kernel(CacheView 
   }
   const UnitBudget u = unit_budget(T, keep, n_min, n_local, n_cap, c.status, b * c.Hkv + h, tid == 0);
   const int M = u.M, n = u.n, F = u.F, nf = u.nf, r = u.r;
-  const int per_warp = ((M + 31) / 32 + kTopnCtaWarps - 1) / kTopnCtaWarps * 32;  // <= 32 kTopnCtaKeys
+  const int per_warp = ((M + 31) / 32 + kTopnCtaWarps - 1) / kTopnCtaWarps * 32;  // <= 32 kKeys (the launch picks kKeys)
   const int w0 = warp * per_warp;
   // bit j: id w0 + 32 j + lane is a candidate (< F) / a forced block taken ([F, F + nf))
   uint32_t cand = 0, forced = 0;
 #pragma unroll
-  for (int j = 0; j < kTopnCtaKeys; ++j) {
+  for (int j = 0; j < kKeys; ++j) {
     const int i = w0 + 32 * j + lane;
     if (32 * j < per_warp) {
       if (i < F) cand |= 1u << j;
@@ -789,12 +790,12 @@ __global__ void __launch_bounds__(kTopnCtaThreads, 2) topn_cta_kernel(CacheView 
   const float* sc = scores + (static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks + w0 + lane;
   pdl_wait();  // the scores
   pdl_launch_dependents();  // after the wait: see the score kernel
-  uint32_t key[kTopnCtaKeys];
+  uint32_t key[kKeys];
 #pragma unroll
-  for (int j = 0; j < kTopnCtaKeys; ++j) key[j] = (cand >> j) & 1u ? score_key(sc[32 * j]) : 0u;
+  for (int j = 0; j < kKeys; ++j) key[j] = (cand >> j) & 1u ? score_key(sc[32 * j]) : 0u;
   uint32_t kmin = 0xFFFFFFFFu, kmax = 0u;
 #pragma unroll
-  for (int j = 0; j < kTopnCtaKeys; ++j)
+  for (int j = 0; j < kKeys; ++j)
     if ((cand >> j) & 1u) {
       kmin = min(kmin, key[j]);
       kmax = max(kmax, key[j]);
@@ -809,7 +810,7 @@ __global__ void __launch_bounds__(kTopnCtaThreads, 2) topn_cta_kernel(CacheView 
   kmin = __reduce_min_sync(0xffffffffu, lane < kTopnCtaWarps ? w_lo[lane] : 0xFFFFFFFFu);
   kmax = __reduce_max_sync(0xffffffffu, lane < kTopnCtaWarps ? w_hi[lane] : 0u);
 #pragma unroll
-  for (int j = 0; j < kTopnCtaKeys; ++j) key[j] -= kmin;  // v = key - min key (candidates only are read)
+  for (int j = 0; j < kKeys; ++j) key[j] -= kmin;  // v = key - min key (candidates only are read)
 
   // ---- radix select of the r-th largest v among blocks [0, F) ----
   uint32_t prefix = 0, pmask = 0;
@@ -822,7 +823,7 @@ __global__ void __launch_bounds__(kTopnCtaThreads, 2) topn_cta_kernel(CacheView 
       int* hb = hist[pass % 3];
       if (tid < 256) hist[(pass + 1) % 3][tid] = 0;
 #pragma unroll
-      for (int j = 0; j < kTopnCtaKeys; ++j)
+      for (int j = 0; j < kKeys; ++j)
         if (((cand >> j) & 1u) && (key[j] & pmask) == prefix) atomicAdd(&hb[(key[j] >> shift) & dmask], 1);
       __syncthreads();  // this pass's histogram is complete
       if (warp == 0) {
@@ -847,7 +848,7 @@ __global__ void __launch_bounds__(kTopnCtaThreads, 2) topn_cta_kernel(CacheView 
   const int take_eq = rem;
   uint32_t gtm = forced, eqm = 0;
 #pragma unroll
-  for (int j = 0; j < kTopnCtaKeys; ++j)
+  for (int j = 0; j < kKeys; ++j)
     if ((cand >> j) & 1u) {
       const uint32_t v = key[j] & pmask;
       if (v > prefix) gtm |= 1u << j;
@@ -868,7 +869,7 @@ __global__ void __launch_bounds__(kTopnCtaThreads, 2) topn_cta_kernel(CacheView 
   int pos = __shfl_sync(0xffffffffu, is - s_l, warp);
   const unsigned below = (1u << lane) - 1u;
 #pragma unroll
-  for (int j = 0; j < kTopnCtaKeys; ++j) {
+  for (int j = 0; j < kKeys; ++j) {
     if (32 * j >= per_warp) break;
     const bool is_eq = (eqm >> j) & 1u;
     const unsigned eqb = __ballot_sync(0xffffffffu, is_eq);
@@ -916,9 +917,18 @@ cudaError_t launch_select(const CacheView& c, const uint16_t* q, double keep, in
                       : launch_score<8, 3>(c, q, scores, sm_count, st, 4);
   if (e != cudaSuccess) return e;
   const size_t smem = select_smem_bytes(c.max_blocks);
-  if (c.max_blocks <= kTopnCtaMaxBlocks)
-    return launch_pdl(topn_cta_kernel, dim3(c.Hkv, c.B), dim3(kTopnCtaThreads), smem, st, c,
+  if (c.max_blocks <= kTopnCtaMaxBlocks) {
+    // key slots per thread for the cache's largest unit: the loops over the
+    // slots unroll to the smallest instantiation that holds them
+    const int slots = ((c.max_blocks + 31) / 32 + kTopnCtaWarps - 1) / kTopnCtaWarps;
+    const auto kernel = slots <= 2   ? topn_cta_kernel<2>
+                        : slots <= 4 ? topn_cta_kernel<4>
+                        : slots <= 6 ? topn_cta_kernel<6>
+                        : slots <= 8 ? topn_cta_kernel<8>
+                                     : topn_cta_kernel<kTopnCtaKeys>;
+    return launch_pdl(kernel, dim3(c.Hkv, c.B), dim3(kTopnCtaThreads), smem, st, c,
                       static_cast<const float*>(scores), keep, n_min, n_local, indices, counts, n_cap);
+  }
   if (smem > 48 * 1024) {
     e = ensure_smem_attr(reinterpret_cast<const void*>(topn_kernel), kTopnSmemMax, 2);
     if (e != cudaSuccess) return e;
