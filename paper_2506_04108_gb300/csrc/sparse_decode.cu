@@ -308,8 +308,15 @@ struct LenAdvance {
 // relative to its own maximum, and the warps' maxima and rows are combined
 // through shared memory.
 constexpr int kMergeWarps = 8;
-constexpr int kMergeLoads = 10;  // partial rows in flight per lane (80 splits in one round)
 
+// kLoads partial rows in flight per lane (8 kLoads splits in one round); the
+// launch picks the smallest instantiation of at least 4 that covers the
+// splits in one round (up to 80; more take further rounds with an online
+// rescale). The 1- and 2-load forms measured slower in the fused decode
+// step although they do less work; with fewer registers, more of the merge
+// CTAs launched early can be placed on each SM beside the decode CTAs, so
+// the merge would run on fewer SMs (the likely cause).
+template <int kLoads>
 __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const float* __restrict__ o_part,
                                                                  const float* __restrict__ lse_part, int splits,
                                                                  uint16_t* __restrict__ out,
@@ -317,7 +324,7 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const float* __
                                                                  const int32_t* __restrict__ active,
                                                                  int rows_per_seq, LenAdvance adv) {
   __shared__ float4 red[kMergeWarps][kHeadDim / 4];
-  __shared__ float wmax[kMergeWarps];
+  __shared__ float wmax[kMergeWarps], wsum[kMergeWarps];
   pdl_launch_dependents();
   pdl_wait();
   const size_t row = blockIdx.x;
@@ -330,15 +337,16 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const float* __
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const float* lp = lse_part + row * splits;
   const float4* op = reinterpret_cast<const float4*>(o_part + row * splits * kHeadDim) + lane;
-  // this warp's splits w + 8 j and their log2-sum-exps, ten of each in
-  // flight together (one pass for up to 80 splits, an online rescale beyond)
+  // this warp's splits w + 8 j and their log2-sum-exps, kLoads of each in
+  // flight together; the warp's weighted sum of rows (acc) and of weights
+  // (l, the normaliser's share) are relative to its running maximum m
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  float m = kNegInf;
-  for (int base = 0; base < splits; base += kMergeWarps * kMergeLoads) {
-    float4 v[kMergeLoads];
-    float ls[kMergeLoads];
+  float m = kNegInf, l = 0.f;
+  for (int base = 0; base < splits; base += kMergeWarps * kLoads) {
+    float4 v[kLoads];
+    float ls[kLoads];
 #pragma unroll
-    for (int j = 0; j < kMergeLoads; ++j) {
+    for (int j = 0; j < kLoads; ++j) {
       const int sp = base + warp + kMergeWarps * j;
       const bool ok = sp < splits;
       v[j] = ok ? op[static_cast<size_t>(sp) * (kHeadDim / 4)] : make_float4(0.f, 0.f, 0.f, 0.f);
@@ -346,20 +354,22 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const float* __
     }
     float mb = m;
 #pragma unroll
-    for (int j = 0; j < kMergeLoads; ++j) mb = fmaxf(mb, ls[j]);
+    for (int j = 0; j < kLoads; ++j) mb = fmaxf(mb, ls[j]);
     const float sc = m == kNegInf ? 0.f : exp2f(m - safe_base(mb));
     acc.x *= sc;
     acc.y *= sc;
     acc.z *= sc;
     acc.w *= sc;
+    l *= sc;
     m = mb;
 #pragma unroll
-    for (int j = 0; j < kMergeLoads; ++j) {
+    for (int j = 0; j < kLoads; ++j) {
       const float w = exp2f(ls[j] - safe_base(m));
       acc.x += w * v[j].x;
       acc.y += w * v[j].y;
       acc.z += w * v[j].z;
       acc.w += w * v[j].w;
+      l += w;
     }
   }
   // acc is this warp's sum relative to its own maximum m: rescale to the CTA's
@@ -371,6 +381,7 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const float* __
   const float sc = m == kNegInf ? 0.f : exp2f(m - safe_base(M));
   acc.x *= sc; acc.y *= sc; acc.z *= sc; acc.w *= sc;
   red[warp][lane] = acc;
+  if (lane == 0) wsum[warp] = l * sc;
   __syncthreads();
   if (warp == 0) {
     float4 t = red[0][lane];
@@ -381,11 +392,10 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const float* __
       t.z += red[w][lane].z;
       t.w += red[w][lane].w;
     }
-    // the normaliser: sum over all splits of exp2(lse - M), lane-strided
+    // the normaliser: the warps' weight sums, relative to M
     float l = 0.f;
-    for (int sp = lane; sp < splits; sp += 32) l += exp2f(lp[sp] - safe_base(M));
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+    for (int w = 0; w < kMergeWarps; ++w) l += wsum[w];
     const float inv = l > 0.f ? 1.f / l : 0.f;
     uint2 packed;
     packed.x = pack_bf16x2(t.x * inv, t.y * inv);
@@ -430,8 +440,12 @@ cudaError_t launch_merge(const float* o_part, const float* lse_part, int rows, i
   LenAdvance adv{nullptr, 0, 0};
   if (advance != nullptr && advance->pending > 0)
     adv = LenAdvance{advance->seq_lens, advance->pending, advance->max_blocks * kBlock};
-  return launch_pdl(merge_kernel, dim3(rows), dim3(kMergeWarps * 32), 0, st, o_part, lse_part, splits, out,
-                    lse_out, active, rows_per_seq, adv);
+  const int per_warp = (splits + kMergeWarps - 1) / kMergeWarps;
+  const auto kernel = per_warp <= 4 ? merge_kernel<4>
+                      : per_warp <= 6 ? merge_kernel<6>
+                                      : merge_kernel<10>;
+  return launch_pdl(kernel, dim3(rows), dim3(kMergeWarps * 32), 0, st, o_part, lse_part, splits, out, lse_out,
+                    active, rows_per_seq, adv);
 }
 
 }  // namespace resa
