@@ -921,8 +921,11 @@ cudaError_t launch_select(const CacheView& c, const uint16_t* q, double keep, in
     // key slots per thread for the cache's largest unit: the loops over the
     // slots unroll to the smallest instantiation that holds them
     const int slots = ((c.max_blocks + 31) / 32 + kTopnCtaWarps - 1) / kTopnCtaWarps;
-    const auto kernel = slots <= 2   ? topn_cta_kernel<2>
+    const auto kernel = slots <= 1   ? topn_cta_kernel<1>
+                        : slots <= 2 ? topn_cta_kernel<2>
+                        : slots <= 3 ? topn_cta_kernel<3>
                         : slots <= 4 ? topn_cta_kernel<4>
+                        : slots <= 5 ? topn_cta_kernel<5>
                         : slots <= 6 ? topn_cta_kernel<6>
                         : slots <= 8 ? topn_cta_kernel<8>
                                      : topn_cta_kernel<kTopnCtaKeys>;
