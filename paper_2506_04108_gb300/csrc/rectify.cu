@@ -337,15 +337,17 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
         }
         float mx;
         {
+          // three-input maxima, four independent chains of 16 keys
           float m4[4];
 #pragma unroll
           for (int y = 0; y < 4; ++y) {
             float v = sv[y];
+            static_assert(kTileKeys == 64, "keys y, y + 4, ..., y + 60");
 #pragma unroll
-            for (int x = y + 4; x < kTileKeys; x += 4) v = fmaxf(v, sv[x]);
-            m4[y] = v;
+            for (int k = 0; k < 7; ++k) v = max3f(v, sv[y + 4 + 8 * k], sv[y + 8 + 8 * k]);
+            m4[y] = fmaxf(v, sv[y + 60]);
           }
-          mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * a.scale_log2;  // scale > 0 keeps the order
+          mx = fmaxf(max3f(m4[0], m4[1], m4[2]), m4[3]) * a.scale_log2;  // scale > 0 keeps the order
         }
         const float m_new = fmaxf(m_used, mx);
         const bool need = m_new > m_used + kRescaleLog2;  // per row
@@ -374,15 +376,23 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
         if (need) m_used = m_new;
         const float nbase = -safe_base(m_used);
         uint32_t w[kTileKeys / 2];  // P row as packed bf16 pairs (keys 2x, 2x + 1)
-        float ls[4] = {0.f, 0.f, 0.f, 0.f};
+        // exponent arguments and row sums two keys per instruction
+        const uint64_t sc2 = pack_f32x2(a.scale_log2, a.scale_log2), nb2 = pack_f32x2(nbase, nbase);
+        uint64_t ls2[2] = {0ull, 0ull};
 #pragma unroll
         for (int x = 0; x < kTileKeys / 2; ++x) {
-          const float p0 = ex2_approx(fmaf(sv[2 * x], a.scale_log2, nbase));
-          const float p1 = ex2_approx(fmaf(sv[2 * x + 1], a.scale_log2, nbase));
-          ls[x & 3] += p0 + p1;
+          float x0, x1;
+          unpack_f32x2(fma_f32x2(pack_f32x2(sv[2 * x], sv[2 * x + 1]), sc2, nb2), x0, x1);
+          const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
+          ls2[x & 1] = add_f32x2(ls2[x & 1], pack_f32x2(p0, p1));
           w[x] = pack_bf16x2(p0, p1);
         }
-        l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+        {
+          float a0, a1, b0, b1;
+          unpack_f32x2(ls2[0], a0, a1);
+          unpack_f32x2(ls2[1], b0, b1);
+          l += (a0 + a1) + (b0 + b1);
+        }
         // P over the S columns it came from (this thread's lane; S is in registers)
         tmem_st32(lane_base + kColS + (buf * kMaxMTiles + mt) * kTileKeys, w);
         tmem_st_wait();
