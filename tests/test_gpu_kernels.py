@@ -190,11 +190,12 @@ def test_select_large_unit():
     check_select_case(cache, Ks, Vs, q, p, maxb, idx, cnt)
 
 
-@pytest.mark.parametrize("M", [6144, 5121])
+@pytest.mark.parametrize("M", [6144, 5121, 4000])
 def test_select_one_cta_at_its_size_bound(M):
     """The one-CTA top-n at the largest cache it serves: 6144 blocks fill all
     twelve key slots of every thread; 5121 blocks leave the last warp with no
-    ids and the one before it with a partial range. Some blocks repeat, so
+    ids and the one before it with a partial range; 4000 blocks take the
+    8-slot instantiation. Some blocks repeat, so
     ties at the boundary are resolved by index."""
     T = M * 16 - 5
     gk = synth.rng(76)
@@ -380,6 +381,8 @@ def run_decode(cache, q_bits, sel_rows, n_cap, p, splits):
 @pytest.mark.parametrize("g,Hkv,lens,nsel,splits", [
     (4, 2, [4100], 26, 0), (7, 4, [2053, 999], 40, 0), (7, 4, [2053, 999], 40, 1), (7, 4, [2053], 40, 7),
     (8, 1, [33], 3, 64), (1, 2, [500], 1, 0), (7, 1, [16 * 300 + 5], 300, 0), (2, 1, [17], 2, 3),
+    (7, 2, [16 * 220 + 3], 200, 100),      # 100 splits: the merge takes two rounds of loads
+    (5, 1, [3000], 100, 16), (3, 2, [1200, 700], 40, 0),
 ])
 def test_sparse_decode_matches_oracle(g, Hkv, lens, nsel, splits):
     Ks, Vs = seq_inputs(10 + g, len(lens), Hkv, lens)
