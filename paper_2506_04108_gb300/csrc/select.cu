@@ -190,20 +190,27 @@ __global__ void __maxnreg__(88) score_kernel(CacheView c, const uint16_t* __rest
     nmine = ncta > warp ? (ncta - warp + kScoreWarps - 1) / kScoreWarps : 0;
   };
   my_range();
+  // the location (sequence, head, first block, blocks) of the piece in each
+  // stage, written by lane 0 when it issues the copy and read by the warp
+  // when it scores the stage, so that a piece is located once
+  __shared__ int4 sh_loc[kScoreWarps][kScoreStages];
   struct Src {
     const uint16_t* p;
     uint32_t bytes;
+    int4 loc;
   };
-  auto piece_src = [&](int k) {  // this warp's k-th piece: its summaries and size
+  auto piece_src = [&](int k) {  // this warp's k-th piece: its summaries, size and location
     int b, h, blk0, nblk;
     locate(c0 + warp + k * kScoreWarps, b, h, blk0, nblk);
     return Src{c.summ + ((static_cast<size_t>(b) * c.Hkv + h) * c.max_blocks + blk0) * 2 * kHeadDim,
-               static_cast<uint32_t>(nblk) * 2 * kHeadDim * 2};
+               static_cast<uint32_t>(nblk) * 2 * kHeadDim * 2, make_int4(b, h, blk0, nblk)};
   };
   auto issue_src = [&](int k, const Src& src) {  // lane 0: piece k into stage (kbase + k) % kScoreStages
-    const uint32_t bar = bar0 + 8 * ((kbase + k) % kScoreStages);
+    const int stage = (kbase + k) % kScoreStages;
+    const uint32_t bar = bar0 + 8 * stage;
+    sh_loc[warp][stage] = src.loc;
     mbar_arrive_expect_tx(bar, src.bytes);
-    bulk_load(ring_s + ((kbase + k) % kScoreStages) * kPieceBytes, src.p, src.bytes, bar);
+    bulk_load(ring_s + stage * kPieceBytes, src.p, src.bytes, bar);
   };
   auto issue = [&](int k) { issue_src(k, piece_src(k)); };
   __syncwarp();  // lane 0's barrier initialisation precedes every lane's use
@@ -232,6 +239,7 @@ __global__ void __maxnreg__(88) score_kernel(CacheView c, const uint16_t* __rest
     kbase = issued_early;
     if (lane == 0)
       for (int k = 0; k < min(kScoreStages, nmine); ++k) issue(k);
+    __syncwarp();  // the stages' locations are visible to the warp
   }
 
   const int ch = lane & 15, half = lane >> 4;  // the appended token: a lane folds 8 dims
@@ -242,8 +250,8 @@ __global__ void __maxnreg__(88) score_kernel(CacheView c, const uint16_t* __rest
   uint4 ka = make_uint4(0, 0, 0, 0), va = ka;  // the appended token's key / value, this lane's 8 dims
   for (int k = 0; k < nmine; ++k) {
     const int st = (kbase + k) % kScoreStages, par = ((kbase + k) / kScoreStages) & 1;
-    int b, h, blk0, nblk;
-    locate(c0 + warp + k * kScoreWarps, b, h, blk0, nblk);
+    const int4 loc = sh_loc[warp][st];
+    const int b = loc.x, h = loc.y, blk0 = loc.z, nblk = loc.w;
     const int unit = b * c.Hkv + h;
     if (unit != cur_unit) {  // pooled query (mean of the group's heads), this lane's 16 dims
       cur_unit = unit;
