@@ -175,14 +175,18 @@ __global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid
     // S^T = K * Q^T
     float sc[4] = {0.f, 0.f, 0.f, 0.f};
     {
+      // two accumulators (even / odd k-steps) halve the dependent MMA chain
+      float sd[4] = {0.f, 0.f, 0.f, 0.f};
       const int key = (lane & 7) + ((lane >> 3) & 1) * 8;
 #pragma unroll
       for (int ks = 0; ks < 8; ++ks) {
         const int chunk = 2 * ks + (lane >> 4);
         uint32_t a0, a1, a2, a3;
         ldsm_x4(kb + (chunk >> 3) * 2048 + sw128(key, chunk & 7), a0, a1, a2, a3);
-        mma_bf16_16816(sc, a0, a1, a2, a3, qb[ks][0], qb[ks][1]);
+        mma_bf16_16816((ks & 1) ? sd : sc, a0, a1, a2, a3, qb[ks][0], qb[ks][1]);
       }
+#pragma unroll
+      for (int i = 0; i < 4; ++i) sc[i] += sd[i];
     }
     const int k0 = lane >> 2;
     float s0 = (k0 < valid) ? sc[0] * a.scale_log2 : kNegInf;
