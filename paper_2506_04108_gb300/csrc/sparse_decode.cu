@@ -32,6 +32,7 @@ constexpr int kStageBytes = 8192;  // K: 2 x 2 KB halves, V: 2 x 2 KB halves
 constexpr int kRingBytes = kWarps * kStages * kStageBytes;
 constexpr int kDecodeSmem = kRingBytes + 1024 /* alignment slack */ + kWarps * kStages * 8;
 constexpr float kNegInf = -__builtin_huge_valf();
+constexpr float kLazyLog2 = 8.f;  // base moves when a score exceeds it by more than 2^8
 
 struct DecodeArgs {
   const uint16_t* q;
@@ -193,28 +194,37 @@ __global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid
     float s1 = (k0 < valid) ? sc[1] * a.scale_log2 : kNegInf;
     float s2 = (k0 + 8 < valid) ? sc[2] * a.scale_log2 : kNegInf;
     float s3 = (k0 + 8 < valid) ? sc[3] * a.scale_log2 : kNegInf;
-    float bm0 = fmaxf(s0, s2), bm1 = fmaxf(s1, s3);
+    // Lazy base: a head's base (m) moves only when one of the block's scores
+    // exceeds it by more than 2^8 (then to the exact running maximum, with O
+    // and l rescaled); otherwise the block needs no cross-lane maximum and no
+    // rescale. P = 2^(s - m) <= 2^8 is exact in range for bf16 and fp32.
+    if (__any_sync(0xffffffffu, s0 > m0 + kLazyLog2 || s2 > m0 + kLazyLog2 || s1 > m1 + kLazyLog2 ||
+                                    s3 > m1 + kLazyLog2)) {
+      float bm0 = fmaxf(s0, s2), bm1 = fmaxf(s1, s3);
 #pragma unroll
-    for (int o = 4; o < 32; o <<= 1) {
-      bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, o));
-      bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, o));
+      for (int o = 4; o < 32; o <<= 1) {
+        bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, o));
+        bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, o));
+      }
+      const float n0 = fmaxf(m0, bm0), n1 = fmaxf(m1, bm1);
+      const float al0 = exp2f(m0 - safe_base(n0)), al1 = exp2f(m1 - safe_base(n1));
+      l0 *= al0;
+      l1 *= al1;
+      m0 = n0;
+      m1 = n1;
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) {
+        acc[mt][0] *= al0;
+        acc[mt][1] *= al1;
+        acc[mt][2] *= al0;
+        acc[mt][3] *= al1;
+      }
     }
-    const float n0 = fmaxf(m0, bm0), n1 = fmaxf(m1, bm1);
-    const float base0 = safe_base(n0), base1 = safe_base(n1);
-    const float al0 = exp2f(m0 - base0), al1 = exp2f(m1 - base1);
+    const float base0 = safe_base(m0), base1 = safe_base(m1);
     const uint32_t x0 = pack_bf16x2(exp2f(s0 - base0), exp2f(s1 - base1));
     const uint32_t x1 = pack_bf16x2(exp2f(s2 - base0), exp2f(s3 - base1));
-    l0 = l0 * al0 + bf16_lo(x0) + bf16_lo(x1);
-    l1 = l1 * al1 + bf16_hi(x0) + bf16_hi(x1);
-    m0 = n0;
-    m1 = n1;
-#pragma unroll
-    for (int mt = 0; mt < 8; ++mt) {
-      acc[mt][0] *= al0;
-      acc[mt][1] *= al1;
-      acc[mt][2] *= al0;
-      acc[mt][3] *= al1;
-    }
+    l0 += bf16_lo(x0) + bf16_lo(x1);
+    l1 += bf16_hi(x0) + bf16_hi(x1);
     const uint32_t pb0 = movmatrix_t(x0), pb1 = movmatrix_t(x1);
     // O^T += V^T * P^T
     {
