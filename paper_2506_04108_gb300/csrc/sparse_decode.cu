@@ -277,14 +277,15 @@ __global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid
   }
   const float fA = LA > 0.f ? exp2f(m0 - safe_base(MA)) / LA : 0.f;
   const float fB = LB > 0.f ? exp2f(m1 - safe_base(MB)) / LB : 0.f;
-  float* red = reinterpret_cast<float*>(smem);  // [warp][8 heads][128] fp32, reuses the ring
+  constexpr int kRedRow = kHeadDim + 4;  // padded: the four heads a warp writes at once fall in distinct banks
+  float* red = reinterpret_cast<float*>(smem);  // [warp][8 heads][kRedRow] fp32, reuses the ring
 #pragma unroll
   for (int mt = 0; mt < 8; ++mt) {
     const int dA = 16 * mt + (lane >> 2), dB = dA + 8;
-    red[(warp * 8 + hA) * kHeadDim + dA] = acc[mt][0] * fA;
-    red[(warp * 8 + hB) * kHeadDim + dA] = acc[mt][1] * fB;
-    red[(warp * 8 + hA) * kHeadDim + dB] = acc[mt][2] * fA;
-    red[(warp * 8 + hB) * kHeadDim + dB] = acc[mt][3] * fB;
+    red[(warp * 8 + hA) * kRedRow + dA] = acc[mt][0] * fA;
+    red[(warp * 8 + hB) * kRedRow + dA] = acc[mt][1] * fB;
+    red[(warp * 8 + hA) * kRedRow + dB] = acc[mt][2] * fA;
+    red[(warp * 8 + hB) * kRedRow + dB] = acc[mt][3] * fB;
   }
   __syncthreads();
   const int t = threadIdx.x;
@@ -293,7 +294,7 @@ __global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid
     for (int dd = t; dd < kHeadDim; dd += kWarps * 32) {  // output dims of this thread
       float v = 0.f;
 #pragma unroll
-      for (int w = 0; w < kWarps; ++w) v += red[(w * 8 + hh) * kHeadDim + dd];
+      for (int w = 0; w < kWarps; ++w) v += red[(w * 8 + hh) * kRedRow + dd];
       a.o_part[(row * a.splits + s) * kHeadDim + dd] = v;
     }
   }

@@ -263,6 +263,31 @@ def test_select_cluster_ties_at_the_boundary(tied, scale, keep):
     assert np.array_equal(idx[0, 0, :n], O.select_blocks(scores, n, 1))
 
 
+@pytest.mark.parametrize("n_tied,n", [(20, 11), (32, 17), (100, 51)])
+def test_select_one_cta_ties_at_the_boundary(n_tied, n):
+    """One-CTA top-n (2,048 blocks, the 32K shape) with the n-th largest
+    score shared by a group of 20, 32 or 100 equal top-scoring blocks (alone
+    in the first radix pass's top bucket): the ids equal the oracle's
+    exactly, ties to the lower ids."""
+    M, g = 2048, 4
+    tied = range(300, 300 + 3 * n_tied, 3)
+    K, V = _tied_unit(M, tied, 4.0, 71)
+    maxb = M + 10
+    cache = H.make_cache([K], [V], g, maxb, compact=True)
+    q = synth.normal_bf16(synth.rng(75), (1, g, 128))
+    keep = n / M  # exact in binary: ceil(M keep) = n
+    p = resa.params(keep, 0, 1)
+    n_cap = resa.resa_max_selected(cache.struct, p)
+    idx, cnt = run_select(cache, q, p, n_cap)
+    assert resa.resa_read_device_error(cache.struct) == (0, 0)
+    st = H.oracle_state(K, V, maxb * 16)
+    _, scores, n_o = O.select_for_group(st, 0, O.widen_bf16(q[0]), O.ResaParams(keep, 0, 1))
+    assert cnt[0, 0] == n_o == n
+    tie = scores[tied[0]]
+    assert np.sum(scores > tie) < n - 1 < np.sum(scores >= tie)  # the boundary lies inside the tied blocks
+    assert np.array_equal(idx[0, 0, :n], O.select_blocks(scores, n, 1))
+
+
 @pytest.mark.parametrize("maxb", [110, 6200])  # one-CTA and cluster top-n
 def test_select_budget_over_cap_is_reported_and_clamped(maxb):
     Ks, Vs = seq_inputs(9, 1, 1, [1600])
