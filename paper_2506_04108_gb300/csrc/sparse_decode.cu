@@ -17,7 +17,8 @@
 //     and accumulates O^T += V^T * P^T with 8 more MMAs (V^T via ldmatrix.trans).
 //   * The 4 warps' (m, l, O) are merged through shared memory; the CTA writes
 //     a normalised partial O (fp32) and its log2-sum-exp for each head.
-// merge_kernel, one CTA per output row: LSE-weighted sum of the split partials.
+// merge_kernel, one CTA per output row: LSE-weighted sum of the split partials
+// (merge_rows_kernel, one warp per row, for calls of many rows and few splits).
 #include <atomic>
 
 #include "resa_device.cuh"
@@ -323,6 +324,7 @@ struct LenAdvance {
 // relative to its own maximum, and the warps' maxima and rows are combined
 // through shared memory.
 constexpr int kMergeWarps = 8;
+constexpr int kRowMergeMinRows = 1024;  // calls with at least this many rows (and <= 16 splits) merge a row per warp
 
 // kLoads partial rows in flight per lane (8 kLoads splits in one round); the
 // launch picks the smallest instantiation of at least 4 that covers the
@@ -420,6 +422,72 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const float* __
   }
 }
 
+// One warp per output row, for calls with many rows and few splits (the
+// rectification's partials: B f Hq rows of a few splits each), where a CTA
+// per row would leave most of its warps idle: lane l holds dims 4l .. 4l + 3
+// of kLoads partial rows in flight and the warp keeps the running maximum,
+// the weighted row sum and the weight sum (an online rescale between rounds
+// when there are more than kLoads splits). No shared memory, no barrier.
+template <int kLoads>
+__global__ void __launch_bounds__(kMergeWarps * 32) merge_rows_kernel(const float* __restrict__ o_part,
+                                                                      const float* __restrict__ lse_part,
+                                                                      int splits, int rows, uint16_t* __restrict__ out,
+                                                                      float* __restrict__ lse_out,
+                                                                      const int32_t* __restrict__ active,
+                                                                      int rows_per_seq, LenAdvance adv) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int lane = threadIdx.x & 31;
+  const size_t row = static_cast<size_t>(blockIdx.x) * kMergeWarps + (threadIdx.x >> 5);
+  if (row >= static_cast<size_t>(rows)) return;
+  if (adv.lens != nullptr && lane == 0 && row % rows_per_seq == 0) {
+    const int b = static_cast<int>(row / rows_per_seq);
+    const int T = adv.lens[b];
+    if (T >= 0 && T + adv.pending <= adv.cap) adv.lens[b] = T + adv.pending;
+  }
+  if (active != nullptr && active[row / rows_per_seq] == 0) return;  // a sequence left out of the call
+  const float* lp = lse_part + row * splits;
+  const float4* op = reinterpret_cast<const float4*>(o_part + row * splits * kHeadDim) + lane;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  float m = kNegInf, l = 0.f;
+  for (int base = 0; base < splits; base += kLoads) {
+    float4 v[kLoads];
+    float ls[kLoads];
+#pragma unroll
+    for (int j = 0; j < kLoads; ++j) {
+      const int sp = base + j;
+      const bool ok = sp < splits;
+      v[j] = ok ? op[static_cast<size_t>(sp) * (kHeadDim / 4)] : make_float4(0.f, 0.f, 0.f, 0.f);
+      ls[j] = ok ? lp[sp] : kNegInf;
+    }
+    float mb = m;
+#pragma unroll
+    for (int j = 0; j < kLoads; ++j) mb = fmaxf(mb, ls[j]);
+    const float sc = m == kNegInf ? 0.f : exp2f(m - safe_base(mb));
+    acc.x *= sc;
+    acc.y *= sc;
+    acc.z *= sc;
+    acc.w *= sc;
+    l *= sc;
+    m = mb;
+#pragma unroll
+    for (int j = 0; j < kLoads; ++j) {
+      const float w = exp2f(ls[j] - safe_base(m));
+      acc.x += w * v[j].x;
+      acc.y += w * v[j].y;
+      acc.z += w * v[j].z;
+      acc.w += w * v[j].w;
+      l += w;
+    }
+  }
+  const float inv = l > 0.f ? 1.f / l : 0.f;
+  uint2 packed;
+  packed.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+  packed.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+  *reinterpret_cast<uint2*>(out + row * kHeadDim + 4 * lane) = packed;
+  if (lse_out != nullptr && lane == 0) lse_out[row] = l > 0.f ? (m + log2f(l)) * 0.69314718055994530942f : kNegInf;
+}
+
 }  // namespace
 
 int decode_ctas_per_sm() {
@@ -455,6 +523,12 @@ cudaError_t launch_merge(const float* o_part, const float* lse_part, int rows, i
   LenAdvance adv{nullptr, 0, 0};
   if (advance != nullptr && advance->pending > 0)
     adv = LenAdvance{advance->seq_lens, advance->pending, advance->max_blocks * kBlock};
+  if (rows >= kRowMergeMinRows && splits <= 16) {
+    // many rows of few splits: a warp per row, all of a row's splits in flight
+    const auto kernel = splits <= 4 ? merge_rows_kernel<4> : splits <= 8 ? merge_rows_kernel<8> : merge_rows_kernel<16>;
+    return launch_pdl(kernel, dim3((rows + kMergeWarps - 1) / kMergeWarps), dim3(kMergeWarps * 32), 0, st, o_part,
+                      lse_part, splits, rows, out, lse_out, active, rows_per_seq, adv);
+  }
   const int per_warp = (splits + kMergeWarps - 1) / kMergeWarps;
   const auto kernel = per_warp <= 4 ? merge_kernel<4>
                       : per_warp <= 6 ? merge_kernel<6>
