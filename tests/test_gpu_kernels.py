@@ -474,6 +474,7 @@ def test_sparse_decode_bad_block_id_is_reported_not_faulted():
 @pytest.mark.parametrize("g,Hkv,lens,f", [
     (4, 2, [4100], 8), (7, 4, [2053, 640], 32), (7, 1, [1000], 16), (7, 1, [777], 64), (8, 2, [64], 64),
     (1, 1, [300], 8), (7, 2, [32], 32),
+    (7, 4, [300, 280, 333, 290, 310, 305], 32),  # 5,376 rows of 5 splits: the merge takes a warp per row
 ])
 def test_rectify_matches_oracle(g, Hkv, lens, f):
     Ks, Vs = seq_inputs(30 + f, len(lens), Hkv, lens)
@@ -542,11 +543,12 @@ def test_chunked_prefill_equals_dense_causal_attention(L, C):
             assert np.array_equal(O.widen_bf16(summ[b, h, :M, 1]), kmax)
 
 
-def test_active_mask_commit_and_rectify():
+@pytest.mark.parametrize("f", [16, 64])  # 384 output rows (a CTA per row) / 1,536 (a warp per row)
+def test_active_mask_commit_and_rectify(f):
     """Continuous batching: only sequences with active[b] != 0 are rectified,
     appended to or overwritten; the others keep their cache, length, block
     keys and output rows, and record no error."""
-    g, Hkv, f = 4, 2, 16
+    g, Hkv = 4, 2
     lens = [700, 333, 1025]
     B = len(lens)
     Ks, Vs = seq_inputs(97, B, Hkv, lens)
