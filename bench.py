@@ -639,15 +639,20 @@ def run_ours(args, w: synth.Workload):
     # timed calls (select and decode stand for their share of decode_step)
     dominant = max((k for k in per_step_us if k != "decode_step"), key=per_step_us.get)
     topn = "topn_cta_kernel" if layers[0].cache.max_blocks <= TOPN_CTA_MAX_BLOCKS else "topn_kernel"
-    kernel, src = {"decode": ("sparse_decode_kernel+merge_kernel", "sparse_decode.cu"),
-                   "select": ("score_kernel+" + topn, "select.cu"),
-                   "rectify": ("rectify_kernel+merge_kernel", "rectify.cu"),
-                   "commit": ("commit_append_kernel", "kv_commit.cu"),
-                   "overwrite": ("commit_overwrite_kernel", "kv_commit.cu")}[dominant]
+    rect_rows = B * f * w.num_q_heads
+    rect_merge = ("merge_rows_kernel" if rect_rows >= ROW_MERGE_MIN_ROWS and
+                  layers[0].resa.resa_rectify_num_splits(layers[0].cache.struct, f) <= ROW_MERGE_MAX_SPLITS
+                  else "merge_kernel")
+    # the call's kernels and the sources they are built from (the merges live in sparse_decode.cu)
+    kernel, src = {"decode": ("sparse_decode_kernel+merge_kernel", ("sparse_decode.cu",)),
+                   "select": ("score_kernel+" + topn, ("select.cu",)),
+                   "rectify": ("rectify_kernel+" + rect_merge, ("rectify.cu", "sparse_decode.cu")),
+                   "commit": ("commit_append_kernel", ("kv_commit.cu",)),
+                   "overwrite": ("commit_overwrite_kernel", ("kv_commit.cu",))}[dominant]
     achieved = algo[dominant] / (mean_us[dominant] * 1e-6) / 1e9
     roofline = {"bound": "hbm", "call": dominant, "kernel": kernel, "achieved": round(achieved, 1), "peak": hbm,
                 "unit": "GB/s", "frac": round(achieved / hbm, 3), "peak_kind": peak_kind,
-                "traffic": profiled_traffic(dominant, w.name, source_hash(src)),
+                "traffic": profiled_traffic(dominant, w.name, source_hash(*src)),
                 "algorithmic_bytes_per_launch": int(algo[dominant]),
                 "timing": "CUDA events around a graph of the step's calls of this kind; per call = total / calls"}
 
@@ -696,6 +701,7 @@ CPU_BASELINE_SECONDS = 10.0  # oracle work timed for cpu_baseline (whole periods
 CPU_BASELINE_ALL_SECONDS = 5.0    # the informational all-cores timing of the same sample
 ORACLE_MAX_REPEATS = 400
 TOPN_CTA_MAX_BLOCKS = 6144  # caches of up to this many blocks per sequence use the one-CTA top-n
+ROW_MERGE_MIN_ROWS, ROW_MERGE_MAX_SPLITS = 1024, 16  # merges of at least this many rows, at most this many splits, take a warp per row
 
 
 E2E_INPUTS = ("q", "k", "v", "rq", "rk", "rv")  # LayerCache device inputs of one period
