@@ -1,6 +1,7 @@
 """Host-side logic of bench.py (CPU only): the algorithmic byte model against
 Eq. 6, the multi-rank aggregation over a world_size-2 gloo group, and the
 timing loop of the CPU baseline."""
+import json
 import math
 import os
 
@@ -107,3 +108,21 @@ def test_clock_summary_keeps_the_timed_window(tmp_path):
     everything = sampler(None)
     assert everything["samples"] == 4 and everything["window"] == "all samples"
     assert everything["reasons"] == ["hw_slowdown"] and everything["sm_mhz"] == 1785.0
+
+
+def test_profiled_traffic_needs_the_current_source_hash(tmp_path, monkeypatch):
+    """The roofline's `traffic` comes from a committed ncu summary only while
+    the kernel sources it was taken from are unchanged (a stale entry gives
+    None); a call built from two sources hashes both."""
+    h_dec = bench.source_hash("sparse_decode.cu")
+    h_rect = bench.source_hash("rectify.cu", "sparse_decode.cu")
+    assert h_rect != bench.source_hash("rectify.cu")
+    table = {"decode": {"w": {"dram_bytes_per_call": 123, "source_hash": h_dec}},
+             "rectify": {"w": {"dram_bytes_per_call": 456, "source_hash": bench.source_hash("rectify.cu")}}}
+    (tmp_path / "profiles").mkdir()
+    (tmp_path / "profiles" / "traffic.json").write_text(json.dumps(table))
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.profiled_traffic("decode", "w", h_dec) == 123
+    assert bench.profiled_traffic("rectify", "w", h_rect) is None  # taken before the merge source was hashed too
+    assert bench.profiled_traffic("select", "w", h_dec) is None
+    assert bench.profiled_traffic("decode", "other workload", h_dec) is None
