@@ -352,6 +352,41 @@ def test_decode_step_equals_commit_select_decode(wide):
         assert np.array_equal(sa[b, :, :M], sf[b, :, :M]), b
 
 
+def test_decode_step_large_batch_equals_commit_select_decode():
+    """Batch 40 at the 28/4 head geometry: 1,120 output rows, merged a row per
+    warp, whose merge also advances seq_lens in the fused step. Ids, counts,
+    outputs and log-sum-exps equal those of the three calls bit for bit, and
+    every length grows by one per step."""
+    B, Hkv, g, steps = 40, 4, 7, 3
+    lens = [int(x) for x in synth.rng(96).integers(1, 400, size=B)]
+    maxb = (max(lens) + steps + 15) // 16 + 2
+    A, F = _decode_step_caches(lens, Hkv, g, maxb, 2, 97)
+    p = resa.params(0.1, 4, 1)
+    n_cap = resa.resa_max_selected(A.struct, p)
+    wa, nb = H.workspace(A, n_cap)
+    wf, _ = H.workspace(F, n_cap)
+    mk = lambda shape, dt: torch.empty(shape, dtype=dt, device="cuda")
+    ia, ifu = mk((B, Hkv, n_cap), torch.int32), mk((B, Hkv, n_cap), torch.int32)
+    ca, cf = mk((B, Hkv), torch.int32), mk((B, Hkv), torch.int32)
+    oa, of = mk((B, g * Hkv, 128), torch.bfloat16), mk((B, g * Hkv, 128), torch.bfloat16)
+    la, lf = mk((B, g * Hkv), torch.float32), mk((B, g * Hkv), torch.float32)
+    gen = synth.rng(98)
+    for t in range(steps):
+        k = H.dev_bf16(synth.normal_bf16(gen, (B, 1, Hkv, 128)))
+        v = H.dev_bf16(synth.normal_bf16(gen, (B, 1, Hkv, 128)))
+        q = H.dev_bf16(synth.normal_bf16(gen, (B, g * Hkv, 128)))
+        resa.resa_commit_kv(A.struct, k, v, 1, False)
+        resa.resa_select_blocks(A.struct, q, p, ia, ca, n_cap, wa, nb)
+        resa.resa_sparse_decode(A.struct, q, ia, ca, n_cap, p, oa, la, 0, wa, nb)
+        resa.resa_decode_step(F.struct, k, v, q, p, ifu, cf, n_cap, of, lf, 0, wf, nb)
+        assert torch.equal(ia, ifu) and torch.equal(ca, cf), t
+        assert np.array_equal(H.host_bits(oa), H.host_bits(of)), t
+        assert np.array_equal(la.cpu().numpy().view(np.uint32), lf.cpu().numpy().view(np.uint32)), t
+    assert resa.resa_read_device_error(A.struct) == (0, 0)
+    assert resa.resa_read_device_error(F.struct) == (0, 0)
+    assert A.seq_lens.cpu().tolist() == F.seq_lens.cpu().tolist() == [T + steps for T in lens]
+
+
 def test_decode_step_sequence_at_capacity():
     """A sequence whose cache is full cannot take the appended token: the
     fused step reports RESA_DEV_SEQ_LEN_RANGE, gives it count 0 and ids -1,
@@ -408,6 +443,7 @@ def run_decode(cache, q_bits, sel_rows, n_cap, p, splits):
     (8, 1, [33], 3, 64), (1, 2, [500], 1, 0), (7, 1, [16 * 300 + 5], 300, 0), (2, 1, [17], 2, 3),
     (7, 2, [16 * 220 + 3], 200, 100),      # 100 splits: the merge takes two rounds of loads
     (5, 1, [3000], 100, 16), (3, 2, [1200, 700], 40, 0),
+    (7, 4, [100 + 7 * i for i in range(37)], 6, 0),  # 1,036 output rows: the merge takes a warp per row
 ])
 def test_sparse_decode_matches_oracle(g, Hkv, lens, nsel, splits):
     Ks, Vs = seq_inputs(10 + g, len(lens), Hkv, lens)
