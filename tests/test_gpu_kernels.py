@@ -190,6 +190,36 @@ def test_select_large_unit():
     check_select_case(cache, Ks, Vs, q, p, maxb, idx, cnt)
 
 
+def test_select_at_the_largest_cache():
+    """One unit of 409,600 blocks (6.55M tokens), the largest page-table row
+    the library accepts: the cluster top-n stages 51,200 keys per CTA (its
+    whole 200 KB). Every block holds one key repeated, so its summary is
+    that key on both sides (checked bit for bit); the ids equal the oracle's
+    up to the near-tie rule."""
+    M, g, Hkv = 409600, 2, 1
+    T = M * 16 - 5
+    keys = synth.normal_bf16(synth.rng(81), (M, 128))
+    pt = synth.page_table(synth.rng(82), 1, M)
+    cache = resa.PagedKVCache(1, g * Hkv, Hkv, M, pt, zero_pools=True)
+    rows = torch.from_numpy(pt[0].astype(np.int64)).cuda()
+    cache.k_pool.view(M, 16, 128)[rows] = H.dev_bf16(keys)[:, None, :].expand(M, 16, 128)
+    cache.seq_lens.fill_(T)
+    resa.resa_update_summaries(cache.struct, 0, -1)
+    summ = H.host_bits(cache.summaries)[0, 0]
+    assert np.array_equal(summ[:, 0], keys) and np.array_equal(summ[:, 1], keys)
+    q = synth.normal_bf16(synth.rng(83), (1, g, 128))
+    p = resa.params(0.05, 128, 1)
+    n_cap = resa.resa_max_selected(cache.struct, p)
+    idx, cnt = run_select(cache, q, p, n_cap)
+    assert resa.resa_read_device_error(cache.struct) == (0, 0)
+    kf = O.widen_bf16(keys)
+    scores = O.quest_scores(O.pooled_query(O.widen_bf16(q[0])), kf, kf)
+    n = O.selection_budget(M, 0.05, 128, 1)
+    assert cnt[0, 0] == n == 20480
+    assert np.all(idx[0, 0, n:] == -1)
+    H.check_selection(idx[0, 0, :n], scores, n, 1)
+
+
 @pytest.mark.parametrize("M", [6144, 5121, 4000])
 def test_select_one_cta_at_its_size_bound(M):
     """The one-CTA top-n at the largest cache it serves: 6144 blocks fill all
