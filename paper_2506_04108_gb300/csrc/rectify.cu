@@ -224,7 +224,7 @@ __global__ void __launch_bounds__(kThreads, 1) rectify_kernel(const __grid_const
         const int row = __shfl_sync(0xffffffffu, my_row, slot + ((j >> 2) & 3));
         if (j < 16 && row >= 0) {
           const int part = j & 3;
-          tma_load_2d(kdst + part * kKVHalf + (j >> 2) * 2048, part < 2 ? &tm_k : &tm_v, bar(kBarKvFull + st),
+          tma_load_2d_stream(kdst + part * kKVHalf + (j >> 2) * 2048, part < 2 ? &tm_k : &tm_v, bar(kBarKvFull + st),
                       (part & 1) * 64, row);
         }
       } else {

@@ -166,12 +166,23 @@ __device__ __forceinline__ bool mbar_wait_polls(uint32_t bar, uint32_t parity, u
 }
 
 // ------------------------------------------------------------------ TMA ---
-// 2-D tiled bulk-tensor load global -> shared, completing on an mbarrier.
-// c0 = innermost coordinate (elements), c1 = row.
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const void* tmap, uint32_t bar, int32_t c0, int32_t c1) {
+// The "stream" copies below carry an L2 evict-first policy (created in the
+// same asm block, so no register stays live across a loop for it). They move
+// data that a call reads once: the K/V tiles of the decode and the
+// rectification, the block summaries of the score kernel. Evicting those
+// first keeps the small tables that every call reads again (page tables,
+// lengths, queries, scores, selected ids, split partials) resident in L2
+// (measured: 32K x 8 decode call 15.66 -> 14.65 us, select 12.2 -> 11.2 us).
+
+// 2-D tiled bulk-tensor load global -> shared of streamed data (L2
+// evict-first), completing on an mbarrier. c0 = innermost coordinate
+// (elements), c1 = row.
+__device__ __forceinline__ void tma_load_2d_stream(uint32_t dst, const void* tmap, uint32_t bar, int32_t c0,
+                                                   int32_t c1) {
   asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%3, %4}], [%2];" ::"r"(dst),
+      "{\n\t.reg .b64 pol;\n\tcreatepolicy.fractional.L2::evict_first.b64 pol, 1.0;\n\t"
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%3, %4}], [%2], pol;\n\t}" ::"r"(dst),
       "l"(tmap), "r"(bar), "r"(c0), "r"(c1)
       : "memory");
 }
@@ -186,12 +197,15 @@ __device__ __forceinline__ void tma_load_4d(uint32_t dst, const void* tmap, uint
       : "memory");
 }
 
-// 1-D bulk copy global -> shared (16-byte aligned addresses, size a multiple
-// of 16), completing on an mbarrier.
-__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
-  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
-               "l"(src), "r"(bytes), "r"(bar)
-               : "memory");
+// 1-D bulk copy global -> shared of streamed data (L2 evict-first; 16-byte
+// aligned addresses, size a multiple of 16), completing on an mbarrier.
+__device__ __forceinline__ void bulk_load_stream(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile(
+      "{\n\t.reg .b64 pol;\n\tcreatepolicy.fractional.L2::evict_first.b64 pol, 1.0;\n\t"
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], pol;"
+      "\n\t}" ::"r"(dst),
+      "l"(src), "r"(bytes), "r"(bar)
+      : "memory");
 }
 
 // Bulk prefetch of [src, src + bytes) into L2 (16-byte aligned, size a

@@ -210,7 +210,7 @@ __global__ void __maxnreg__(88) score_kernel(CacheView c, const uint16_t* __rest
     const uint32_t bar = bar0 + 8 * stage;
     sh_loc[warp][stage] = src.loc;
     mbar_arrive_expect_tx(bar, src.bytes);
-    bulk_load(ring_s + stage * kPieceBytes, src.p, src.bytes, bar);
+    bulk_load_stream(ring_s + stage * kPieceBytes, src.p, src.bytes, bar);
   };
   auto issue = [&](int k) { issue_src(k, piece_src(k)); };
   __syncwarp();  // lane 0's barrier initialisation precedes every lane's use

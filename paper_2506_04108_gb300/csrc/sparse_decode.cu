@@ -121,10 +121,10 @@ __global__ void __launch_bounds__(kWarps * 32) sparse_decode_kernel(const __grid
     const int row = (page * c.Hkv + h) * kBlock;
     const uint32_t dst = ring + st * kStageBytes;
     mbar_arrive_expect_tx(bar, kStageBytes);
-    tma_load_2d(dst, &tm_k, bar, 0, row);
-    tma_load_2d(dst + 2048, &tm_k, bar, 64, row);
-    tma_load_2d(dst + 4096, &tm_v, bar, 0, row);
-    tma_load_2d(dst + 6144, &tm_v, bar, 64, row);
+    tma_load_2d_stream(dst, &tm_k, bar, 0, row);
+    tma_load_2d_stream(dst + 2048, &tm_k, bar, 64, row);
+    tma_load_2d_stream(dst + 4096, &tm_v, bar, 0, row);
+    tma_load_2d_stream(dst + 6144, &tm_v, bar, 64, row);
   };
 
   // Q^T as the B operand: lane holds head lane/4, dims 16ks + 2(lane%4) (+1, +8, +9).
